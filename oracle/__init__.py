@@ -1,0 +1,200 @@
+"""LookME CPU oracle: TEST INFRASTRUCTURE ONLY.
+
+A plain, slow, double-precision restatement of the hierarchical two-level
+lookup and sparse injection of arXiv 2607.16305 (Sec. "Image Embedding
+Hierarchical Two-Level Lookup", Sec. "Sparse Injection").  The arithmetic is
+in ``lookme_oracle.c``; this module compiles it with gcc, loads it with
+ctypes and marshals numpy arrays.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import this package.  The CUDA library never does, and the two
+share no code.
+
+Every function takes float32 arrays that hold the exact input values (bf16
+inputs widened to float32 are exact) and computes in float64.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "lookme_oracle.c")
+_LIB = os.path.join(_HERE, "liblookme_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False, src: str = _SRC, out: str = _LIB) -> str:
+    """Compile the C oracle into a shared library (gcc -O2 -fopenmp)."""
+    if not force and os.path.exists(out) and os.path.getmtime(out) >= os.path.getmtime(src):
+        return out
+    tmp = out + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", src, "-o", tmp, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, out)
+    return out
+
+
+_I64 = ctypes.c_int64
+_I32 = ctypes.c_int32
+_P = ctypes.c_void_p
+_D = ctypes.c_double
+
+_SIGS = {
+    "lkm_centroids": [_I64, _I64, _I64, _P, _P],
+    "lkm_route": [_I64, _I64, _I64, _P, _P, _P, _P, _P, _P, _P],
+    "lkm_primitives": [_I64, _I64, _I64, _I32, _P, _P, _P, _P, _P, _P, _P, _P, _P],
+    "lkm_weights_for": [_I64, _I64, _I64, _I32, _P, _P, _P, _P, _P, _P],
+    "lkm_select": [_I64, _P, _I32, _P, _D, _P, _P, _P],
+    "lkm_inject": [_I64, _I64, _I64, _I32, _P, _P, _P, _P, _P, _P, _I32, _P, _P],
+    "lkm_round_bf16": [_I64, _P, _P],
+}
+
+
+def load(path: str | None = None):
+    """Build (if needed) and load the oracle library.  A path loads that file instead."""
+    global _lib
+    if path is not None:
+        lib = ctypes.CDLL(path)
+        for name, argtypes in _SIGS.items():
+            fn = getattr(lib, name)
+            fn.argtypes = argtypes
+            fn.restype = None
+        return lib
+    with _lock:
+        if _lib is None:
+            _lib = load(build())
+    return _lib
+
+
+def _f32(a):
+    return np.ascontiguousarray(np.asarray(a, dtype=np.float32))
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data
+
+
+def _blocks(blocks, block_of_scene, n_scene):
+    """Scene blocks [n_blocks, P, d] plus the scene -> block map (identity if None)."""
+    blocks = _f32(blocks)
+    if block_of_scene is None:
+        block_of_scene = np.arange(n_scene, dtype=np.int64)
+    return blocks, np.ascontiguousarray(block_of_scene, dtype=np.int64)
+
+
+class Oracle:
+    """numpy front end to the C oracle.  ``lib`` may be a mutated build (tests)."""
+
+    def __init__(self, lib=None):
+        self.lib = lib if lib is not None else load()
+
+    def centroids(self, keys):
+        """e_img[s] = mean over primitives of K[s] (Level-1, first equation)."""
+        keys = _f32(keys)
+        S, P, dk = keys.shape
+        out = np.empty((S, dk), np.float64)
+        self.lib.lkm_centroids(S, P, dk, _ptr(keys), _ptr(out))
+        return out
+
+    def route(self, q, cent, bias=None):
+        """Level-1 routing.  Returns dict(scene, score, gap1, qnorm)."""
+        q, cent = _f32(q), _f32(cent)
+        N, dk = q.shape
+        S = cent.shape[0]
+        bias = None if bias is None else _f32(bias)
+        scene = np.empty(N, np.int32)
+        score, gap1, qnorm = (np.empty(N, np.float64) for _ in range(3))
+        self.lib.lkm_route(N, S, dk, _ptr(q), _ptr(cent), _ptr(bias),
+                           _ptr(scene), _ptr(score), _ptr(gap1), _ptr(qnorm))
+        return dict(scene=scene, score=score, gap1=gap1, qnorm=qnorm)
+
+    def primitives(self, q, scene, key_blocks, top_k, block_of_scene=None, n_scene=None):
+        """Level-2 scoring, top-k and softmax.  Returns dict(prim, weight, logit, gap_k, gap_adj)."""
+        q = _f32(q)
+        N, dk = q.shape
+        kb = np.asarray(key_blocks)
+        P = kb.shape[1]
+        kb, bos = _blocks(kb, block_of_scene, n_scene if n_scene is not None else kb.shape[0])
+        scene = np.ascontiguousarray(scene, dtype=np.int32)
+        if N and (scene.min() < 0 or scene.max() >= bos.shape[0] or (bos[scene] < 0).any()):
+            raise ValueError("a token's scene block is missing")
+        if not 1 <= top_k <= min(P, 64):
+            raise ValueError("top_k out of range")
+        prim = np.empty((N, top_k), np.int32)
+        weight, logit = np.empty((N, top_k), np.float64), np.empty((N, top_k), np.float64)
+        gap_k, gap_adj = np.empty(N, np.float64), np.empty(N, np.float64)
+        self.lib.lkm_primitives(N, P, dk, top_k, _ptr(q), _ptr(scene), _ptr(kb), _ptr(bos),
+                                _ptr(prim), _ptr(weight), _ptr(logit), _ptr(gap_k), _ptr(gap_adj))
+        return dict(prim=prim, weight=weight, logit=logit, gap_k=gap_k, gap_adj=gap_adj)
+
+    def weights_for(self, q, scene, prim, key_blocks, block_of_scene=None, n_scene=None):
+        """Softmax weights of a given primitive set (conditional oracle)."""
+        q = _f32(q)
+        N, dk = q.shape
+        kb = np.asarray(key_blocks)
+        P = kb.shape[1]
+        kb, bos = _blocks(kb, block_of_scene, n_scene if n_scene is not None else kb.shape[0])
+        prim = np.ascontiguousarray(prim, dtype=np.int32)
+        top_k = prim.shape[1]
+        if top_k > 64:
+            raise ValueError("top_k out of range")
+        scene = np.ascontiguousarray(scene, dtype=np.int32)
+        weight = np.empty((N, top_k), np.float64)
+        self.lib.lkm_weights_for(N, P, dk, top_k, _ptr(q), _ptr(scene), _ptr(prim),
+                                 _ptr(kb), _ptr(bos), _ptr(weight))
+        return weight
+
+    def select(self, priority, keep_ratio, seg_off=None):
+        """Top-r token selection per segment.  Returns dict(mask, pi_r, pi_r1, seg_off)."""
+        pr = np.ascontiguousarray(priority, dtype=np.float64)
+        N = pr.shape[0]
+        if seg_off is None:
+            seg_off = [0, N]
+        seg_off = np.ascontiguousarray(seg_off, dtype=np.int64)
+        n_seg = seg_off.shape[0] - 1
+        mask = np.empty(N, np.uint8)
+        pi_r, pi_r1 = np.empty(n_seg, np.float64), np.empty(n_seg, np.float64)
+        self.lib.lkm_select(N, _ptr(pr), n_seg, _ptr(seg_off), float(keep_ratio),
+                            _ptr(mask), _ptr(pi_r), _ptr(pi_r1))
+        return dict(mask=mask, pi_r=pi_r, pi_r1=pi_r1, seg_off=seg_off)
+
+    def inject(self, scene, prim, weight, mask, value_blocks, hidden, block_of_scene=None, n_scene=None):
+        """h' = h + sum_j w_j V[scene, prim_j] on masked rows of every layer.  Returns float64 [L,N,dv]."""
+        hidden = _f32(hidden)
+        if hidden.ndim == 2:
+            hidden = hidden[None]
+        L, N, dv = hidden.shape
+        vb = np.asarray(value_blocks)
+        P = vb.shape[1]
+        vb, bos = _blocks(vb, block_of_scene, n_scene if n_scene is not None else vb.shape[0])
+        prim = np.ascontiguousarray(prim, dtype=np.int32)
+        top_k = prim.shape[1]
+        weight = np.ascontiguousarray(weight, dtype=np.float64)
+        mask = np.ascontiguousarray(mask, dtype=np.uint8)
+        scene = np.ascontiguousarray(scene, dtype=np.int32)
+        sel_scenes = scene[mask.astype(bool)]
+        if sel_scenes.size and (bos[sel_scenes] < 0).any():
+            raise ValueError("a selected token's value block is missing")
+        out = np.empty((L, N, dv), np.float64)
+        self.lib.lkm_inject(N, P, dv, top_k, _ptr(scene), _ptr(prim), _ptr(weight), _ptr(mask),
+                            _ptr(vb), _ptr(bos), L, _ptr(hidden), _ptr(out))
+        return out
+
+    def round_bf16(self, x):
+        """Round-to-nearest-even to bf16; returns the uint16 bit patterns."""
+        x = np.ascontiguousarray(x, dtype=np.float64)
+        out = np.empty(x.shape, np.uint16)
+        self.lib.lkm_round_bf16(x.size, _ptr(x), _ptr(out))
+        return out
+
+
+def bf16_bits_to_f32(bits):
+    """Widen bf16 bit patterns (uint16) to float32 values (exact)."""
+    b = np.ascontiguousarray(bits, dtype=np.uint16).astype(np.uint32) << 16
+    return b.view(np.float32)
