@@ -1,0 +1,205 @@
+/*
+ * lookme.h - C ABI of the LookME lookup + sparse-injection library (GB300, sm_103a).
+ *
+ * LookME (arXiv 2607.16305) enhances a vision-language model's hidden states
+ * with rows retrieved from a large external table.  The image and cross-modal
+ * pathways look up continuous embeddings in two levels (Sec. "Image Embedding
+ * Hierarchical Two-Level Lookup"):
+ *   level 1  scene_t = argmax_s ( cos(q_t, e_img[s]) + b_s )
+ *   level 2  z_tp = q_t . K[scene_t, p] / sqrt(d_k) for every primitive p of
+ *            that scene, I_t = top-k of z_t, w_t = softmax(z_t[I_t]),
+ *            R_t = sum_j w_tj * V[scene_t, I_tj, :]
+ * and inject R only into the hidden rows of the highest-priority tokens
+ * (Sec. "Sparse Injection"), reusing one lookup across the neighbouring
+ * layers that share a table (Sec. "Inter-Layer Sparse Activation").
+ *
+ * Conventions for every entry point
+ *   - All pointers are plain addresses.  "device" means CUDA device memory of
+ *     the table's device (or host memory the device can address); "host"
+ *     means ordinary CPU memory.  Layouts are row-major and dense.
+ *   - The element type of queries, centroids, keys, values and hidden states
+ *     is the table's dtype (bf16 = IEEE bfloat16 bit patterns, or fp32).
+ *     Indices are int32, weights, norms and priorities fp32.
+ *   - All work is asynchronous on the given stream (a cudaStream_t; NULL is
+ *     the legacy default stream).  No entry point synchronises the stream
+ *     unless its comment says so.  Results are valid once the stream has
+ *     reached the point of the call.
+ *   - The caller owns every buffer it passes; the library never frees or
+ *     keeps caller memory past the call (except the table storage it owns).
+ *   - Errors are return codes; nothing throws or aborts across the ABI.
+ *     lookme_last_error() gives a thread-local message for the last failure.
+ *     An asynchronous CUDA error seen by a later call is returned as
+ *     LOOKME_ERR_CUDA and makes the table unusable (sticky).
+ *   - One table may be used from one stream at a time.
+ */
+#ifndef LOOKME_H
+#define LOOKME_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    LOOKME_OK = 0,
+    LOOKME_ERR_INVALID_ARG = 1,  /* an argument failed validation; nothing was launched */
+    LOOKME_ERR_CUDA = 2,         /* a CUDA call failed (sticky on the table) */
+    LOOKME_ERR_OOM = 3,          /* a device or pinned-host allocation failed */
+    LOOKME_ERR_TIMEOUT = 4,      /* a bounded device-side wait gave up (see lookme_device_status) */
+    LOOKME_ERR_STATE = 5,        /* call out of order (e.g. lookup before every scene is loaded) */
+    LOOKME_ERR_UNSUPPORTED = 6   /* valid request this build does not handle */
+} lookme_status;
+
+typedef enum { LOOKME_BF16 = 0, LOOKME_FP32 = 1 } lookme_dtype;
+
+/* Where the keys and values of a table live.  Centroids always live in HBM.
+ *   DEVICE       keys and values in HBM.
+ *   HOST_STAGED  keys and values in pinned host memory (the paper's
+ *                partitioned storage with on-demand loading, Sec. "Level-2:
+ *                scene-primitive retrieval", last sentence): each lookup
+ *                copies the key blocks of the routed scenes into an HBM slot
+ *                cache on a side stream, and the injection reads the selected
+ *                value rows straight from host memory. */
+typedef enum { LOOKME_RES_DEVICE = 0, LOOKME_RES_HOST_STAGED = 1 } lookme_residency;
+
+typedef void* lookme_stream; /* cudaStream_t */
+
+/* Shape of a two-level table E_img in R^{N_s x N_p x d_e} (Sec. "Two-level
+ * embedding table"), split into keys (scored) and values (injected).  Setting
+ * d_key == d_value and passing the same array for both recovers the paper's
+ * single table. */
+typedef struct {
+    int64_t n_scenes;     /* N_s >= 1 */
+    int64_t n_prims;      /* N_p >= 1 (primitives per scene) */
+    int64_t d_key;        /* key / query width d_k >= 1 (bf16: multiple of 8; fp32: multiple of 4) */
+    int64_t d_value;      /* value / hidden width >= 1 (bf16: multiple of 8; fp32: multiple of 4) */
+    int32_t dtype;        /* lookme_dtype */
+    int32_t residency;    /* lookme_residency */
+    int32_t device;       /* CUDA device ordinal */
+    int32_t reserved0;    /* must be 0 */
+    int64_t max_tokens;   /* scratch is sized for this many tokens per call; 0 = grow on demand */
+    int64_t stage_slots;  /* HOST_STAGED: scenes the HBM slot cache holds (0 = n_scenes) */
+} lookme_table_desc;
+
+typedef struct lookme_table lookme_table; /* opaque, owned by the library */
+
+/* Limits of this build. */
+#define LOOKME_MAX_TOP_K 64        /* top_k <= min(n_prims, 64) */
+#define LOOKME_MAX_LAYERS 64       /* layers sharing one table per inject call */
+#define LOOKME_MAX_SEGMENTS 1024   /* token-selection segments per inject call */
+#define LOOKME_MAX_SCENES 49152    /* n_scenes (bucketing keeps one counter per scene on chip) */
+#define LOOKME_MAX_PRIMS 2048      /* n_prims (level-2 keeps one logit per primitive on chip) */
+#define LOOKME_MAX_DKEY 2048       /* d_key */
+
+/* Create a table on desc->device.  Allocates the table storage (HBM, or
+ * pinned host for HOST_STAGED), the centroids and, if desc->max_tokens > 0,
+ * the per-call scratch.  *out receives the handle; on failure *out is NULL.
+ * Errors: INVALID_ARG (bad shape or limits), OOM, CUDA. */
+lookme_status lookme_table_create(const lookme_table_desc* desc, lookme_table** out);
+
+/* Free everything the table owns.  Synchronises the device first.  NULL is a no-op. */
+lookme_status lookme_table_destroy(lookme_table* table);
+
+/* Copy scenes [scene_begin, scene_begin + n) into the table (Sec. "Two-level
+ * embedding table").
+ *   centroids  [n][d_key] scene-centred embeddings e_img, or NULL: then each
+ *              centroid is the mean of its scene's keys (Sec. "Level-1: scene
+ *              retrieval", first equation), accumulated in fp32 and stored
+ *              in the table dtype.
+ *   keys       [n][n_prims][d_key]     (required)
+ *   values     [n][n_prims][d_value]   (required)
+ *   bias       [n] fp32 routing bias b (Sec. "Level-1", second equation) or
+ *              NULL for 0.  A table with any nonzero bias routes by
+ *              cos + b; without bias by cos alone.
+ *   src_on_device  1 if the sources are device memory, 0 if host memory.
+ * The sources may be reused once the stream reaches the end of the call.
+ * Errors: INVALID_ARG (range, NULL keys/values), CUDA. */
+lookme_status lookme_load_scenes(lookme_table* table, int64_t scene_begin, int64_t n,
+                                 const void* centroids, const void* keys, const void* values,
+                                 const float* bias, int src_on_device, lookme_stream stream);
+
+/* Two-level lookup for n_tokens queries (Sec. "Image Embedding Hierarchical
+ * Two-Level Lookup"; the cross-modal pathway is the same call with the
+ * decoder output as queries):
+ *   queries     device [n_tokens][d_key]
+ *   scene_out   device [n_tokens] int32: level-1 scene (ties: lowest index)
+ *   prim_out    device [n_tokens][top_k] int32: primitives of that scene by
+ *               descending z (ties: lower index)
+ *   weight_out  device [n_tokens][top_k] fp32: softmax over the selected z
+ *   qnorm_out   device [n_tokens] fp32 ||q_t||_2, or NULL (the table keeps
+ *               its own copy for lookme_inject's default priority)
+ * Every token is looked up; selection happens in lookme_inject.
+ * Errors: INVALID_ARG, STATE (a scene not loaded yet, or scratch would have to
+ * grow while the stream is being captured), OOM, CUDA. */
+lookme_status lookme_lookup(lookme_table* table, const void* queries, int64_t n_tokens, int32_t top_k,
+                            int32_t* scene_out, int32_t* prim_out, float* weight_out, float* qnorm_out,
+                            lookme_stream stream);
+
+/* Sparse injection (Sec. "Sparse Injection", S(R) = g * f(R[g]) with f the
+ * identity, and Sec. "Inter-Layer Sparse Activation" with the same gate and
+ * R reused by every layer that shares the table):
+ *   scene, prim, weight   device outputs of lookme_lookup for these tokens
+ *   priority   device [n_tokens] fp32 gate signal, or NULL for the query
+ *              norms of this table's most recent lookup (which must have had
+ *              n_tokens tokens)
+ *   seg_offsets  HOST [n_seg + 1] int64, 0 = off[0] <= ... <= off[n_seg] =
+ *              n_tokens, or NULL for one segment.  Segment i keeps its
+ *              r_i = floor(len_i * keep_ratio) tokens of largest priority
+ *              (ties: lower token index); keep_ratio in [0, 1].
+ *   hidden     HOST array of n_layers device pointers, each [n_tokens][d_value]
+ *              in the table dtype, updated in place: every kept row gets
+ *              + sum_j w_tj V[scene_t, prim_tj, :] (accumulated in fp32,
+ *              rounded once); every other row is left untouched.
+ *   mask_out   device [n_tokens] uint8 (1 = kept) or NULL
+ *   sel_out    device [sum r_i] int32 kept token ids (ascending within each
+ *              segment, segments in order) or NULL
+ * Errors: INVALID_ARG, STATE, OOM, CUDA. */
+lookme_status lookme_inject(lookme_table* table, const int32_t* scene, const int32_t* prim,
+                            const float* weight, int64_t n_tokens, int32_t top_k,
+                            const float* priority, const int64_t* seg_offsets, int32_t n_seg,
+                            double keep_ratio, void* const* hidden, int32_t n_layers,
+                            uint8_t* mask_out, int32_t* sel_out, lookme_stream stream);
+
+/* Size the per-call scratch for up to max_tokens tokens now, so that later
+ * calls (for example under CUDA graph capture) never allocate.  Synchronous. */
+lookme_status lookme_reserve(lookme_table* table, int64_t max_tokens);
+
+/* Statistics of the table's most recent lookup, read back synchronously on
+ * the given stream: routed scenes, level-2 work items, largest bucket. */
+typedef struct {
+    int64_t n_tokens;
+    int32_t n_routed_scenes;  /* distinct scenes that received a token */
+    int32_t n_work_items;     /* level-2 work items (scene, token chunk) */
+    int64_t staged_bytes;     /* HOST_STAGED: key bytes copied host -> HBM */
+} lookme_lookup_stats;
+lookme_status lookme_last_lookup_stats(lookme_table* table, lookme_lookup_stats* out, lookme_stream stream);
+
+/* Device status word of the table (bit 0: a bounded wait inside a kernel
+ * gave up; the kernel then skipped its remaining work).  Synchronises the
+ * stream.  reset != 0 clears it afterwards. */
+lookme_status lookme_device_status(lookme_table* table, uint32_t* status, int reset, lookme_stream stream);
+
+/* Number of CUDA kernels this table has launched since creation. */
+uint64_t lookme_launch_count(const lookme_table* table);
+
+/* Per-kernel tracing.  While enabled, every kernel the table launches is
+ * bracketed by two CUDA events on its stream.  lookme_trace_read
+ * synchronises those events and copies out up to max records (kernel id and
+ * milliseconds), then clears the log.  lookme_kernel_name maps an id to a name. */
+typedef struct {
+    int32_t kernel;
+    float ms;
+} lookme_trace_record;
+lookme_status lookme_trace_enable(lookme_table* table, int enable);
+lookme_status lookme_trace_read(lookme_table* table, lookme_trace_record* out, int32_t max, int32_t* n_out);
+const char* lookme_kernel_name(int32_t kernel);
+
+const char* lookme_status_string(lookme_status status);
+const char* lookme_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LOOKME_H */

@@ -47,6 +47,7 @@ _D = ctypes.c_double
 
 _SIGS = {
     "lkm_centroids": [_I64, _I64, _I64, _P, _P],
+    "lkm_query_norms": [_I64, _I64, _P, _P],
     "lkm_route": [_I64, _I64, _I64, _P, _P, _P, _P, _P, _P, _P],
     "lkm_primitives": [_I64, _I64, _I64, _I32, _P, _P, _P, _P, _P, _P, _P, _P, _P],
     "lkm_weights_for": [_I64, _I64, _I64, _I32, _P, _P, _P, _P, _P, _P],
@@ -100,6 +101,13 @@ class Oracle:
         S, P, dk = keys.shape
         out = np.empty((S, dk), np.float64)
         self.lib.lkm_centroids(S, P, dk, _ptr(keys), _ptr(out))
+        return out
+
+    def query_norms(self, q):
+        """||q_t||_2 in float64 (the default token-selection priority)."""
+        q = _f32(q)
+        out = np.empty(q.shape[0], np.float64)
+        self.lib.lkm_query_norms(q.shape[0], q.shape[1], _ptr(q), _ptr(out))
         return out
 
     def route(self, q, cent, bias=None):

@@ -56,6 +56,16 @@ static double row_norm(const float* x, int64_t n)
     return sqrt(acc);
 }
 
+/* ||q_t||_2 of every query: the default gate priority of the token
+ * selection (Sec. "Intra-Layer Sparse Activation", priority read as the
+ * query norm).  The same value lkm_route reports. */
+void lkm_query_norms(int64_t N, int64_t dk, const float* q, double* qnorm)
+{
+#pragma omp parallel for schedule(static)
+    for (int64_t t = 0; t < N; ++t)
+        qnorm[t] = row_norm(q + t * dk, dk);
+}
+
 /* Level-1 routing: scene_t = argmax_s ( cos(q_t, e_img[s]) + b_s )
  * (Sec. "Level-1: scene retrieval", second equation).
  * Outputs per token: the scene, its score, the gap between the best and the

@@ -1,0 +1,170 @@
+// Shared declarations of the LookME CUDA library: element helpers, argmax key
+// packing, kernel ids and the launch wrappers each kernel file defines.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "lookme.h"
+
+namespace lookme {
+
+// ---------------------------------------------------------------- kernel ids
+enum KernelId : int32_t {
+    KID_PREP = 0,        // K0: ||q||, argmax reset
+    KID_ROUTE_TC = 1,    // K1: level-1 scores on tcgen05 + fused argmax
+    KID_ROUTE_SIMT = 2,  // K1: level-1 scores on CUDA cores (fp32 tables, odd shapes)
+    KID_BUCKET = 3,      // K2: counting sort of tokens by scene + work list
+    KID_SCORE = 4,       // K3: level-2 key scoring + top-k + softmax
+    KID_SELECT = 5,      // K5: top-r token selection per segment
+    KID_INJECT = 6,      // K4: gather + weighted sum + residual add
+    KID_STAGE = 7,       // K6: host -> HBM staging of routed key blocks
+    KID_CENTROID = 8,    // load-time: centroid = mean of keys
+    KID_CNORM = 9,       // load-time: 1 / ||centroid||
+    KID_COUNT
+};
+
+// Device status bits (table status word).
+constexpr uint32_t STATUS_WAIT_TIMEOUT = 1u;
+
+// ------------------------------------------------------------ element access
+__device__ __forceinline__ float to_f32(float x) { return x; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+// 16 bytes -> floats: 8 bf16 or 4 fp32.
+template <typename T> struct Vec16;
+template <> struct Vec16<__nv_bfloat16> {
+    static constexpr int N = 8;
+    __device__ __forceinline__ static void unpack(const uint4& v, float* f) {
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            f[2 * i] = __uint_as_float(w[i] << 16);
+            f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+        }
+    }
+    __device__ __forceinline__ static uint4 pack(const float* f) {
+        uint32_t w[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            __nv_bfloat162 h = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
+            w[i] = *reinterpret_cast<uint32_t*>(&h);
+        }
+        return make_uint4(w[0], w[1], w[2], w[3]);
+    }
+};
+template <> struct Vec16<float> {
+    static constexpr int N = 4;
+    __device__ __forceinline__ static void unpack(const uint4& v, float* f) {
+        f[0] = __uint_as_float(v.x);
+        f[1] = __uint_as_float(v.y);
+        f[2] = __uint_as_float(v.z);
+        f[3] = __uint_as_float(v.w);
+    }
+    __device__ __forceinline__ static uint4 pack(const float* f) {
+        return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]), __float_as_uint(f[2]),
+                          __float_as_uint(f[3]));
+    }
+};
+
+// -------------------------------------------------------- argmax key packing
+// A 64-bit key whose unsigned order is (score ascending, scene descending), so
+// that atomicMax keeps the highest score and, among equal scores, the lowest
+// scene index.  Key 0 means "no candidate".
+__device__ __forceinline__ uint32_t orderable(float f) {
+    uint32_t u = __float_as_uint(f == 0.0f ? 0.0f : f);  // -0 and +0 compare equal
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ unsigned long long pack_argmax(float score, uint32_t scene) {
+    return ((unsigned long long)orderable(score) << 32) | (unsigned long long)(0xFFFFFFFFu - scene);
+}
+__device__ __forceinline__ int32_t unpack_scene(unsigned long long key, int64_t n_scenes) {
+    uint32_t s = 0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull);
+    return (key == 0ull || s >= (uint64_t)n_scenes) ? 0 : (int32_t)s;
+}
+
+// Work item of level 2: tokens perm[begin, begin + count) all routed to
+// `scene`; `slot` is the scene's index in the routed-scene list (and its HBM
+// slot when keys are staged).
+struct WorkItem {
+    int32_t scene, begin, count, slot;
+};
+
+// ------------------------------------------------------------ launch params
+struct LaunchCtx {
+    cudaStream_t stream;
+    int num_sms;
+};
+
+// K0
+cudaError_t launch_prep(const LaunchCtx& c, int dtype, const void* q, int64_t N, int dk, float* qnorm,
+                        float* qnorm_out, unsigned long long* best);
+// K1 (tcgen05, bf16, d_k <= 512).  tmap_q is the CUtensorMap of the queries
+// (box 64 x 128); tmap_c[i] the centroids' map with box 64 x (64 << i).
+constexpr int kRouteTcMaxDk = 512;
+cudaError_t launch_route_tc(const LaunchCtx& c, const void* tmap_q, const void* const tmap_c[3], int64_t N,
+                            int64_t S, int dk, const float* inv_cnorm, const float* bias, const float* qnorm,
+                            unsigned long long* best, uint32_t* status);
+// K1 (CUDA cores)
+cudaError_t launch_route_simt(const LaunchCtx& c, int dtype, const void* q, const void* cent, int64_t N,
+                              int64_t S, int dk, const float* inv_cnorm, const float* bias, const float* qnorm,
+                              unsigned long long* best);
+// K2
+constexpr int kTokensPerItem = 8;
+cudaError_t launch_bucket(const LaunchCtx& c, const unsigned long long* best, int64_t N, int64_t S,
+                          int32_t* scene_out, int32_t* perm, WorkItem* work, int32_t* routed, int32_t* counters);
+// K3
+struct ScoreArgs {
+    int dtype;
+    const void* q;
+    const void* keys;     // [S or slots][P][dk]
+    int64_t P;
+    int dk;
+    int top_k;
+    float scale;          // 1 / sqrt(d_k)
+    const WorkItem* work;
+    const int32_t* n_work;
+    const int32_t* perm;
+    int use_slots;        // index key blocks by WorkItem::slot instead of ::scene
+    int32_t* prim_out;
+    float* weight_out;
+    uint32_t* status;
+};
+cudaError_t launch_score(const LaunchCtx& c, const ScoreArgs& a);
+// K5
+cudaError_t launch_select(const LaunchCtx& c, const float* priority, int64_t N, const int64_t* seg_off_host,
+                          int n_seg, double keep_ratio, uint8_t* mask, int32_t* sel);
+// K4
+struct InjectArgs {
+    int dtype;
+    const void* values;   // [S][P][dv] (device or host-mapped)
+    int64_t P;
+    int dv;
+    int top_k;
+    const int32_t* scene;
+    const int32_t* prim;
+    const float* weight;
+    const int32_t* sel;
+    int64_t n_sel;
+    int64_t N;
+    int64_t S;
+    int n_layers;
+    void* hidden[LOOKME_MAX_LAYERS];
+};
+cudaError_t launch_inject(const LaunchCtx& c, const InjectArgs& a);
+// K6
+cudaError_t launch_stage(const LaunchCtx& c, const void* keys_host_mapped, void* slots, int64_t block_bytes,
+                         int64_t n_slots, const int32_t* routed, const int32_t* counters);
+
+// Raise the dynamic shared-memory limits of the kernels that need more than
+// 48 KB (per device; call with the device current).
+cudaError_t configure_route_kernels();
+cudaError_t configure_bucket_kernel();
+cudaError_t configure_score_kernels();
+// load-time
+cudaError_t launch_centroid_mean(const LaunchCtx& c, int dtype, const void* keys, int64_t n, int64_t P, int dk,
+                                 void* cent);
+cudaError_t launch_inv_cnorm(const LaunchCtx& c, int dtype, const void* cent, int64_t n, int dk, float* inv_cnorm);
+
+}  // namespace lookme

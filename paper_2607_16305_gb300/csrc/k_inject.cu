@@ -1,0 +1,234 @@
+// Sparse injection (Sec. "Sparse Injection" and "Inter-Layer Sparse Activation").
+//
+// K5 select: the intra-layer gate as top-r selection.  In each segment the
+//   r = floor(len * keep_ratio) tokens of largest priority are kept (ties:
+//   lower token index).  One CTA per segment finds the r-th largest priority
+//   with a 4-pass, 8-bit radix select over order-preserving integer keys,
+//   keeps every token above it and the first tokens equal to it, and compacts
+//   the kept ids in ascending order.
+// K4 inject: for every kept token t, R_t = sum_j w_tj V[scene_t, prim_tj, :]
+//   accumulated in fp32 from 16-byte vector loads, then h_l[t] += R_t for every
+//   layer l sharing the table, rounded once to the hidden dtype.  Rows that are
+//   not kept are never touched.
+#include "common.cuh"
+
+namespace lookme {
+
+namespace k5 {
+constexpr int kThreads = 1024;
+
+struct Params {
+    const float* priority;
+    uint8_t* mask;
+    int32_t* sel;
+    double keep_ratio;
+    int n_seg;
+    int64_t off[LOOKME_MAX_SEGMENTS + 1];
+};
+
+__device__ __forceinline__ uint32_t prio_key(float f) { return orderable(f); }
+
+// Block-wide exclusive scan of one int (1024 threads).
+__device__ int block_excl_scan(int v, int& total, int* buf) {
+    const int lane = threadIdx.x % 32, warp = threadIdx.x / 32;
+    int inc = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int n = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+        if (lane >= o) inc += n;
+    }
+    if (lane == 31) buf[warp] = inc;
+    __syncthreads();
+    if (warp == 0) {
+        const int w = buf[lane];
+        int wi = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int n = __shfl_up_sync(0xFFFFFFFFu, wi, o);
+            if (lane >= o) wi += n;
+        }
+        buf[lane] = wi - w;
+        if (lane == 31) buf[32] = wi;
+    }
+    __syncthreads();
+    const int r = buf[warp] + inc - v;
+    total = buf[32];
+    __syncthreads();
+    return r;
+}
+}  // namespace k5
+
+__global__ void __launch_bounds__(k5::kThreads, 1) k5_select(const __grid_constant__ k5::Params p) {
+    using namespace k5;
+    __shared__ int hist[256];
+    __shared__ int scan_buf[33];
+    __shared__ uint32_t sh_prefix;
+    __shared__ int sh_remaining;
+    const int seg = blockIdx.x;
+    const int64_t b = p.off[seg], len = p.off[seg + 1] - p.off[seg];
+    const int64_t r = (int64_t)floor((double)len * p.keep_ratio);
+    int64_t sel_base = 0;
+    for (int i = 0; i < seg; ++i) sel_base += (int64_t)floor((double)(p.off[i + 1] - p.off[i]) * p.keep_ratio);
+    const int tid = threadIdx.x;
+
+    uint32_t prefix = 0, pmask = 0;
+    int remaining = (int)r;
+    if (r > 0 && r < len) {
+        for (int shift = 24; shift >= 0; shift -= 8) {
+            for (int i = tid; i < 256; i += kThreads) hist[i] = 0;
+            __syncthreads();
+            for (int64_t i = tid; i < len; i += kThreads) {
+                const uint32_t k = prio_key(p.priority[b + i]);
+                if ((k & pmask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1);
+            }
+            __syncthreads();
+            if (tid == 0) {
+                int above = 0, d = 255;
+                for (; d > 0; --d) {
+                    if (above + hist[d] >= remaining) break;
+                    above += hist[d];
+                }
+                sh_prefix = prefix | ((uint32_t)d << shift);
+                sh_remaining = remaining - above;
+            }
+            __syncthreads();
+            prefix = sh_prefix;
+            remaining = sh_remaining;
+            pmask |= 255u << shift;
+            __syncthreads();
+        }
+    }
+    // Keep: key > threshold, or key == threshold among the first `remaining` in token order.
+    const uint32_t thr = prefix;
+    int eq_seen = 0, kept_seen = 0;
+    for (int64_t i0 = 0; i0 < len; i0 += kThreads) {
+        const int64_t i = i0 + tid;
+        int is_eq = 0, keep = 0;
+        if (i < len) {
+            if (r >= len) {
+                keep = 1;
+            } else if (r > 0) {
+                const uint32_t k = prio_key(p.priority[b + i]);
+                keep = k > thr;
+                is_eq = k == thr;
+            }
+        }
+        int eq_total;
+        const int eq_rank = block_excl_scan(is_eq, eq_total, scan_buf);
+        if (is_eq && eq_seen + eq_rank < remaining) keep = 1;
+        int kept_total;
+        const int kept_rank = block_excl_scan(keep, kept_total, scan_buf);
+        if (i < len) {
+            if (p.mask) p.mask[b + i] = (uint8_t)keep;
+            if (keep) p.sel[sel_base + kept_seen + kept_rank] = (int32_t)(b + i);
+        }
+        eq_seen += eq_total;
+        kept_seen += kept_total;
+    }
+}
+
+cudaError_t launch_select(const LaunchCtx& c, const float* priority, int64_t N, const int64_t* seg_off_host,
+                          int n_seg, double keep_ratio, uint8_t* mask, int32_t* sel) {
+    if (N == 0 || n_seg == 0) return cudaSuccess;
+    k5::Params p;
+    p.priority = priority;
+    p.mask = mask;
+    p.sel = sel;
+    p.keep_ratio = keep_ratio;
+    p.n_seg = n_seg;
+    for (int i = 0; i <= n_seg; ++i) p.off[i] = seg_off_host ? seg_off_host[i] : (i == 0 ? 0 : N);
+    k5_select<<<n_seg, k5::kThreads, 0, c.stream>>>(p);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- K4 inject
+namespace k4 {
+constexpr int kThreads = 128;
+
+struct Params {
+    const void* values;
+    int64_t P;
+    int dv;
+    int top_k;
+    const int32_t* scene;
+    const int32_t* prim;
+    const float* weight;
+    const int32_t* sel;
+    int64_t N;
+    int64_t S;
+    int n_layers;
+    void* hidden[LOOKME_MAX_LAYERS];
+};
+}  // namespace k4
+
+template <typename T>
+__global__ void __launch_bounds__(k4::kThreads) k4_inject(const __grid_constant__ k4::Params p) {
+    constexpr int EPC = Vec16<T>::N;
+    __shared__ const uint4* rows[LOOKME_MAX_TOP_K];
+    __shared__ float w[LOOKME_MAX_TOP_K];
+    const int64_t t = p.sel[blockIdx.x];
+    const int64_t s = min(max((int64_t)p.scene[t], (int64_t)0), p.S - 1);
+    for (int j = threadIdx.x; j < p.top_k; j += blockDim.x) {
+        const int64_t pr = min(max((int64_t)p.prim[t * p.top_k + j], (int64_t)0), p.P - 1);
+        rows[j] = reinterpret_cast<const uint4*>(reinterpret_cast<const T*>(p.values) + (s * p.P + pr) * p.dv);
+        w[j] = p.weight[t * p.top_k + j];
+    }
+    __syncthreads();
+    const int chunks = p.dv / EPC;
+    for (int ch = threadIdx.x; ch < chunks; ch += blockDim.x) {
+        float acc[EPC];
+#pragma unroll
+        for (int e = 0; e < EPC; ++e) acc[e] = 0.f;
+        int j = 0;
+        for (; j + 4 <= p.top_k; j += 4) {
+            uint4 v[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) v[u] = __ldg(rows[j + u] + ch);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                float f[EPC];
+                Vec16<T>::unpack(v[u], f);
+#pragma unroll
+                for (int e = 0; e < EPC; ++e) acc[e] = fmaf(w[j + u], f[e], acc[e]);
+            }
+        }
+        for (; j < p.top_k; ++j) {
+            float f[EPC];
+            Vec16<T>::unpack(__ldg(rows[j] + ch), f);
+#pragma unroll
+            for (int e = 0; e < EPC; ++e) acc[e] = fmaf(w[j], f[e], acc[e]);
+        }
+        for (int l = 0; l < p.n_layers; ++l) {
+            uint4* h = reinterpret_cast<uint4*>(reinterpret_cast<T*>(p.hidden[l]) + t * p.dv) + ch;
+            float f[EPC];
+            Vec16<T>::unpack(*h, f);
+#pragma unroll
+            for (int e = 0; e < EPC; ++e) f[e] += acc[e];
+            *h = Vec16<T>::pack(f);
+        }
+    }
+}
+
+cudaError_t launch_inject(const LaunchCtx& c, const InjectArgs& a) {
+    if (a.n_sel == 0) return cudaSuccess;
+    k4::Params p;
+    p.values = a.values;
+    p.P = a.P;
+    p.dv = a.dv;
+    p.top_k = a.top_k;
+    p.scene = a.scene;
+    p.prim = a.prim;
+    p.weight = a.weight;
+    p.sel = a.sel;
+    p.N = a.N;
+    p.S = a.S;
+    p.n_layers = a.n_layers;
+    for (int l = 0; l < a.n_layers; ++l) p.hidden[l] = a.hidden[l];
+    if (a.dtype == LOOKME_BF16)
+        k4_inject<__nv_bfloat16><<<(unsigned)a.n_sel, k4::kThreads, 0, c.stream>>>(p);
+    else
+        k4_inject<float><<<(unsigned)a.n_sel, k4::kThreads, 0, c.stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace lookme

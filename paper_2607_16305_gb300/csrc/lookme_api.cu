@@ -1,0 +1,656 @@
+// Host runtime of the LookME library: the C ABI declared in lookme.h.
+//
+// A table owns its storage (HBM, or pinned host memory plus an HBM slot
+// cache), its centroids with their inverse norms, an optional routing bias and
+// the per-call scratch.  Every entry point validates its arguments on the host
+// before touching the device, switches to the table's device for the duration
+// of the call, enqueues kernels on the caller's stream and never synchronises
+// it (except the calls documented as synchronous).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+
+using namespace lookme;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+lookme_status fail(lookme_status st, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return st;
+}
+
+const char* kKernelNames[KID_COUNT] = {"prep", "route_tc", "route_simt", "bucket", "score",
+                                       "select", "inject", "stage", "centroid_mean", "inv_cnorm"};
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point, so the
+// library does not link libcuda directly.
+PFN_cuTensorMapEncodeTiled_v12000 get_encode_tiled() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        cudaDriverEntryPointQueryResult q;
+        void* p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// 2-D bf16 tensor map over a row-major [rows][cols] matrix, 128-byte swizzle,
+// box of 64 columns x box_rows rows; out-of-bounds elements read as zero.
+bool encode_bf16_2d(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int box_rows) {
+    auto fn = get_encode_tiled();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)(cols * 2)};
+    cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Restores the caller's current device on scope exit.
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = false;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) return;
+        ok = (prev == dev) || cudaSetDevice(dev) == cudaSuccess;
+    }
+    ~DeviceGuard() {
+        int cur;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+struct TraceEntry {
+    int32_t kernel;
+    cudaEvent_t start, stop;
+};
+
+}  // namespace
+
+struct lookme_table {
+    lookme_table_desc d{};
+    size_t esz = 2;
+    int num_sms = 0;
+    bool tc_route = false;  // level 1 on tcgen05
+
+    // storage
+    void* keys = nullptr;       // device, or device-mapped pinned host
+    void* values = nullptr;     // device, or device-mapped pinned host
+    void* keys_host = nullptr;  // pinned host allocations (HOST_STAGED)
+    void* values_host = nullptr;
+    void* slots = nullptr;      // HBM slot cache of staged key blocks
+    int64_t n_slots = 0;
+    void* cent = nullptr;
+    float* inv_cnorm = nullptr;
+    float* bias = nullptr;
+    bool has_bias = false;
+    CUtensorMap tmap_c[3];
+    std::vector<uint8_t> loaded;
+    int64_t n_loaded = 0;
+
+    // scratch
+    int64_t cap = 0;
+    void* scratch = nullptr;
+    unsigned long long* best = nullptr;
+    float* qnorm = nullptr;
+    int32_t* perm = nullptr;
+    WorkItem* work = nullptr;
+    int32_t* routed = nullptr;
+    int32_t* counters = nullptr;  // n_work, n_routed, max bucket
+    int32_t* sel = nullptr;
+    uint8_t* mask = nullptr;
+    uint32_t* status = nullptr;   // persistent device status word
+    int64_t last_tokens = -1;
+    int64_t last_staged_bytes = 0;
+
+    lookme_status sticky = LOOKME_OK;
+    uint64_t launches = 0;
+
+    bool trace = false;
+    std::vector<TraceEntry> trace_log;
+    std::vector<cudaEvent_t> event_pool;
+};
+
+namespace {
+
+lookme_status cuda_fail(lookme_table* t, cudaError_t e, const char* what) {
+    if (t) t->sticky = LOOKME_ERR_CUDA;
+    return fail(LOOKME_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+cudaEvent_t pool_event(lookme_table* t) {
+    if (!t->event_pool.empty()) {
+        cudaEvent_t e = t->event_pool.back();
+        t->event_pool.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+}
+
+bool capturing(cudaStream_t s) {
+    cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(s, &st) != cudaSuccess) return false;
+    return st != cudaStreamCaptureStatusNone;
+}
+
+// Runs one kernel launch: counts it, brackets it with trace events if tracing.
+template <typename F>
+lookme_status launch(lookme_table* t, cudaStream_t s, int32_t kid, F&& fn) {
+    const bool tr = t->trace && !capturing(s);
+    TraceEntry te{kid, nullptr, nullptr};
+    if (tr) {
+        te.start = pool_event(t);
+        te.stop = pool_event(t);
+        cudaEventRecord(te.start, s);
+    }
+    cudaError_t e = fn();
+    if (e != cudaSuccess) return cuda_fail(t, e, kKernelNames[kid]);
+    ++t->launches;
+    if (tr) {
+        cudaEventRecord(te.stop, s);
+        t->trace_log.push_back(te);
+    }
+    return LOOKME_OK;
+}
+
+lookme_status check_table(const lookme_table* t) {
+    if (!t) return fail(LOOKME_ERR_INVALID_ARG, "table is NULL");
+    if (t->sticky != LOOKME_OK) return fail(t->sticky, "table is unusable after an earlier CUDA error");
+    return LOOKME_OK;
+}
+
+void free_scratch(lookme_table* t) {
+    if (t->scratch) cudaFree(t->scratch);
+    t->scratch = nullptr;
+    t->cap = 0;
+}
+
+lookme_status ensure_scratch(lookme_table* t, int64_t n, cudaStream_t s) {
+    if (n <= t->cap && t->scratch) return LOOKME_OK;
+    if (s && capturing(s))
+        return fail(LOOKME_ERR_STATE, "scratch must grow to %lld tokens while the stream is captured; call "
+                    "lookme_reserve first", (long long)n);
+    const int64_t cap = n > 0 ? n : 1;
+    const int64_t S = t->d.n_scenes;
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        const size_t o = off;
+        off = align_up(off + bytes, 256);
+        return o;
+    };
+    const size_t o_best = take(cap * sizeof(unsigned long long));
+    const size_t o_qnorm = take(cap * sizeof(float));
+    const size_t o_perm = take(cap * sizeof(int32_t));
+    const size_t o_work = take((cap + S) * sizeof(WorkItem));
+    const size_t o_routed = take(S * sizeof(int32_t));
+    const size_t o_counters = take(4 * sizeof(int32_t));
+    const size_t o_sel = take(cap * sizeof(int32_t));
+    const size_t o_mask = take(cap);
+    void* buf = nullptr;
+    if (cudaDeviceSynchronize() != cudaSuccess || cudaMalloc(&buf, off) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(LOOKME_ERR_OOM, "scratch allocation of %zu bytes failed", off);
+    }
+    free_scratch(t);
+    char* b = static_cast<char*>(buf);
+    t->scratch = buf;
+    t->cap = cap;
+    t->best = reinterpret_cast<unsigned long long*>(b + o_best);
+    t->qnorm = reinterpret_cast<float*>(b + o_qnorm);
+    t->perm = reinterpret_cast<int32_t*>(b + o_perm);
+    t->work = reinterpret_cast<WorkItem*>(b + o_work);
+    t->routed = reinterpret_cast<int32_t*>(b + o_routed);
+    t->counters = reinterpret_cast<int32_t*>(b + o_counters);
+    t->sel = reinterpret_cast<int32_t*>(b + o_sel);
+    t->mask = reinterpret_cast<uint8_t*>(b + o_mask);
+    t->last_tokens = -1;
+    if (cudaMemset(buf, 0, off) != cudaSuccess) return cuda_fail(t, cudaGetLastError(), "scratch memset");
+    return LOOKME_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+void destroy_table(lookme_table* t) {
+    if (!t) return;
+    for (auto& te : t->trace_log) {
+        cudaEventDestroy(te.start);
+        cudaEventDestroy(te.stop);
+    }
+    for (auto e : t->event_pool) cudaEventDestroy(e);
+    free_scratch(t);
+    if (t->d.residency == LOOKME_RES_DEVICE) {
+        if (t->keys) cudaFree(t->keys);
+        if (t->values) cudaFree(t->values);
+    } else {
+        if (t->keys_host) cudaFreeHost(t->keys_host);
+        if (t->values_host) cudaFreeHost(t->values_host);
+        if (t->slots) cudaFree(t->slots);
+    }
+    if (t->cent) cudaFree(t->cent);
+    if (t->inv_cnorm) cudaFree(t->inv_cnorm);
+    if (t->bias) cudaFree(t->bias);
+    if (t->status) cudaFree(t->status);
+    delete t;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* lookme_status_string(lookme_status s) {
+    switch (s) {
+        case LOOKME_OK: return "ok";
+        case LOOKME_ERR_INVALID_ARG: return "invalid argument";
+        case LOOKME_ERR_CUDA: return "CUDA error";
+        case LOOKME_ERR_OOM: return "out of memory";
+        case LOOKME_ERR_TIMEOUT: return "device wait timed out";
+        case LOOKME_ERR_STATE: return "call out of order";
+        case LOOKME_ERR_UNSUPPORTED: return "unsupported";
+    }
+    return "unknown status";
+}
+
+const char* lookme_last_error(void) { return g_last_error.c_str(); }
+
+const char* lookme_kernel_name(int32_t k) { return (k >= 0 && k < KID_COUNT) ? kKernelNames[k] : "?"; }
+
+lookme_status lookme_table_create(const lookme_table_desc* desc, lookme_table** out) {
+    if (!out) return fail(LOOKME_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    if (!desc) return fail(LOOKME_ERR_INVALID_ARG, "desc is NULL");
+    const lookme_table_desc& d = *desc;
+    if (d.dtype != LOOKME_BF16 && d.dtype != LOOKME_FP32) return fail(LOOKME_ERR_INVALID_ARG, "bad dtype %d", d.dtype);
+    if (d.residency != LOOKME_RES_DEVICE && d.residency != LOOKME_RES_HOST_STAGED)
+        return fail(LOOKME_ERR_INVALID_ARG, "bad residency %d", d.residency);
+    if (d.reserved0 != 0) return fail(LOOKME_ERR_INVALID_ARG, "reserved0 must be 0");
+    if (d.n_scenes < 1 || d.n_scenes > LOOKME_MAX_SCENES)
+        return fail(LOOKME_ERR_INVALID_ARG, "n_scenes %lld outside [1, %d]", (long long)d.n_scenes, LOOKME_MAX_SCENES);
+    if (d.n_prims < 1 || d.n_prims > LOOKME_MAX_PRIMS)
+        return fail(LOOKME_ERR_INVALID_ARG, "n_prims %lld outside [1, %d]", (long long)d.n_prims, LOOKME_MAX_PRIMS);
+    if (d.d_key < 1 || d.d_key > LOOKME_MAX_DKEY)
+        return fail(LOOKME_ERR_INVALID_ARG, "d_key %lld outside [1, %d]", (long long)d.d_key, LOOKME_MAX_DKEY);
+    if (d.d_value < 1) return fail(LOOKME_ERR_INVALID_ARG, "d_value must be >= 1");
+    const int vec = d.dtype == LOOKME_BF16 ? 8 : 4;
+    if (d.d_key % vec || d.d_value % vec)
+        return fail(LOOKME_ERR_INVALID_ARG, "d_key and d_value must be multiples of %d for this dtype", vec);
+    if (d.max_tokens < 0 || d.stage_slots < 0) return fail(LOOKME_ERR_INVALID_ARG, "negative size");
+    if ((int64_t)d.n_scenes * d.n_prims > ((int64_t)1 << 31) - 1)
+        return fail(LOOKME_ERR_INVALID_ARG, "n_scenes * n_prims must fit in int32");
+
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || d.device < 0 || d.device >= ndev) {
+        cudaGetLastError();
+        return fail(LOOKME_ERR_INVALID_ARG, "device %d not available (%d devices)", d.device, ndev);
+    }
+    DeviceGuard guard(d.device);
+    if (!guard.ok) return fail(LOOKME_ERR_CUDA, "cannot select device %d", d.device);
+
+    lookme_table* t = new lookme_table();
+    t->d = d;
+    t->esz = d.dtype == LOOKME_BF16 ? 2 : 4;
+    cudaDeviceGetAttribute(&t->num_sms, cudaDevAttrMultiProcessorCount, d.device);
+    t->tc_route = d.dtype == LOOKME_BF16 && d.d_key <= kRouteTcMaxDk;
+    // Validation switch: LOOKME_ROUTE=simt routes bf16 tables on the CUDA-core
+    // kernel too, so the two level-1 kernels can be checked against each other.
+    if (const char* env = getenv("LOOKME_ROUTE")) {
+        if (strcmp(env, "simt") == 0) t->tc_route = false;
+    }
+    t->loaded.assign(d.n_scenes, 0);
+
+    cudaError_t e;
+    if ((e = configure_route_kernels()) != cudaSuccess || (e = configure_bucket_kernel()) != cudaSuccess ||
+        (e = configure_score_kernels()) != cudaSuccess) {
+        destroy_table(t);
+        return fail(LOOKME_ERR_CUDA, "kernel configuration: %s", cudaGetErrorString(e));
+    }
+
+    const size_t S = d.n_scenes, P = d.n_prims;
+    const size_t kbytes = S * P * d.d_key * t->esz, vbytes = S * P * d.d_value * t->esz;
+    bool ok = true;
+    if (d.residency == LOOKME_RES_DEVICE) {
+        ok = cudaMalloc(&t->keys, kbytes) == cudaSuccess && cudaMalloc(&t->values, vbytes) == cudaSuccess;
+    } else {
+        ok = cudaHostAlloc(&t->keys_host, kbytes, cudaHostAllocMapped | cudaHostAllocPortable) == cudaSuccess &&
+             cudaHostAlloc(&t->values_host, vbytes, cudaHostAllocMapped | cudaHostAllocPortable) == cudaSuccess &&
+             cudaHostGetDevicePointer(&t->keys, t->keys_host, 0) == cudaSuccess &&
+             cudaHostGetDevicePointer(&t->values, t->values_host, 0) == cudaSuccess;
+        t->n_slots = d.stage_slots > 0 ? d.stage_slots : d.n_scenes;
+        ok = ok && cudaMalloc(&t->slots, (size_t)t->n_slots * P * d.d_key * t->esz) == cudaSuccess;
+    }
+    ok = ok && cudaMalloc(&t->cent, align_up(S * d.d_key * t->esz, 256)) == cudaSuccess &&
+         cudaMalloc(&t->inv_cnorm, align_up(S * sizeof(float), 256)) == cudaSuccess &&
+         cudaMalloc(&t->bias, align_up(S * sizeof(float), 256)) == cudaSuccess &&
+         cudaMalloc(&t->status, 256) == cudaSuccess;
+    if (!ok) {
+        cudaGetLastError();
+        destroy_table(t);
+        return fail(LOOKME_ERR_OOM, "table allocation failed (%zu key bytes, %zu value bytes)", kbytes, vbytes);
+    }
+    if (cudaMemset(t->bias, 0, S * sizeof(float)) != cudaSuccess ||
+        cudaMemset(t->inv_cnorm, 0, align_up(S * sizeof(float), 256)) != cudaSuccess ||
+        cudaMemset(t->status, 0, 256) != cudaSuccess) {
+        destroy_table(t);
+        return fail(LOOKME_ERR_CUDA, "table initialisation failed");
+    }
+    if (t->tc_route) {
+        for (int i = 0; i < 3; ++i) {
+            if (!encode_bf16_2d(&t->tmap_c[i], t->cent, d.n_scenes, d.d_key, 64 << i)) {
+                destroy_table(t);
+                return fail(LOOKME_ERR_CUDA, "cuTensorMapEncodeTiled failed for the centroids");
+            }
+        }
+    }
+    if (d.max_tokens > 0) {
+        lookme_status st = ensure_scratch(t, d.max_tokens, nullptr);
+        if (st != LOOKME_OK) {
+            destroy_table(t);
+            return st;
+        }
+    }
+    if (cudaDeviceSynchronize() != cudaSuccess) {
+        destroy_table(t);
+        return fail(LOOKME_ERR_CUDA, "table creation: %s", cudaGetErrorString(cudaGetLastError()));
+    }
+    *out = t;
+    return LOOKME_OK;
+}
+
+lookme_status lookme_table_destroy(lookme_table* t) {
+    if (!t) return LOOKME_OK;
+    DeviceGuard guard(t->d.device);
+    cudaDeviceSynchronize();
+    destroy_table(t);
+    return LOOKME_OK;
+}
+
+lookme_status lookme_reserve(lookme_table* t, int64_t max_tokens) {
+    lookme_status st = check_table(t);
+    if (st != LOOKME_OK) return st;
+    if (max_tokens < 0) return fail(LOOKME_ERR_INVALID_ARG, "max_tokens < 0");
+    DeviceGuard guard(t->d.device);
+    return ensure_scratch(t, max_tokens, nullptr);
+}
+
+lookme_status lookme_load_scenes(lookme_table* t, int64_t scene_begin, int64_t n, const void* centroids,
+                                 const void* keys, const void* values, const float* bias, int src_on_device,
+                                 lookme_stream stream) {
+    lookme_status st = check_table(t);
+    if (st != LOOKME_OK) return st;
+    const lookme_table_desc& d = t->d;
+    if (n < 0 || scene_begin < 0 || scene_begin + n > d.n_scenes)
+        return fail(LOOKME_ERR_INVALID_ARG, "scene range [%lld, %lld) outside [0, %lld)", (long long)scene_begin,
+                    (long long)(scene_begin + n), (long long)d.n_scenes);
+    if (!keys || !values) return fail(LOOKME_ERR_INVALID_ARG, "keys and values are required");
+    if (n == 0) return LOOKME_OK;
+    (void)src_on_device;  // copies use unified addressing and work for either source
+    DeviceGuard guard(d.device);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    LaunchCtx ctx{s, t->num_sms};
+    const size_t P = d.n_prims;
+    const size_t krow = P * d.d_key * t->esz, vrow = P * d.d_value * t->esz;
+    char* kdst = static_cast<char*>(d.residency == LOOKME_RES_DEVICE ? t->keys : t->keys_host);
+    char* vdst = static_cast<char*>(d.residency == LOOKME_RES_DEVICE ? t->values : t->values_host);
+    cudaError_t e;
+    if ((e = cudaMemcpyAsync(kdst + scene_begin * krow, keys, n * krow, cudaMemcpyDefault, s)) != cudaSuccess)
+        return cuda_fail(t, e, "copy keys");
+    if ((e = cudaMemcpyAsync(vdst + scene_begin * vrow, values, n * vrow, cudaMemcpyDefault, s)) != cudaSuccess)
+        return cuda_fail(t, e, "copy values");
+    char* cdst = static_cast<char*>(t->cent) + scene_begin * d.d_key * t->esz;
+    if (centroids) {
+        if ((e = cudaMemcpyAsync(cdst, centroids, n * d.d_key * t->esz, cudaMemcpyDefault, s)) != cudaSuccess)
+            return cuda_fail(t, e, "copy centroids");
+    } else {
+        const char* ksrc = static_cast<const char*>(t->keys) + scene_begin * krow;  // device view of the stored keys
+        st = launch(t, s, KID_CENTROID,
+                    [&] { return launch_centroid_mean(ctx, d.dtype, ksrc, n, d.n_prims, (int)d.d_key, cdst); });
+        if (st != LOOKME_OK) return st;
+    }
+    st = launch(t, s, KID_CNORM, [&] {
+        return launch_inv_cnorm(ctx, d.dtype, cdst, n, (int)d.d_key, t->inv_cnorm + scene_begin);
+    });
+    if (st != LOOKME_OK) return st;
+    if (bias) {
+        if ((e = cudaMemcpyAsync(t->bias + scene_begin, bias, n * sizeof(float), cudaMemcpyDefault, s)) !=
+            cudaSuccess)
+            return cuda_fail(t, e, "copy bias");
+        t->has_bias = true;
+    }
+    for (int64_t i = scene_begin; i < scene_begin + n; ++i) {
+        if (!t->loaded[i]) {
+            t->loaded[i] = 1;
+            ++t->n_loaded;
+        }
+    }
+    return LOOKME_OK;
+}
+
+lookme_status lookme_lookup(lookme_table* t, const void* queries, int64_t N, int32_t top_k, int32_t* scene_out,
+                            int32_t* prim_out, float* weight_out, float* qnorm_out, lookme_stream stream) {
+    lookme_status st = check_table(t);
+    if (st != LOOKME_OK) return st;
+    const lookme_table_desc& d = t->d;
+    if (N < 0 || N > INT32_MAX / 2) return fail(LOOKME_ERR_INVALID_ARG, "n_tokens %lld out of range", (long long)N);
+    if (top_k < 1 || top_k > LOOKME_MAX_TOP_K || top_k > d.n_prims)
+        return fail(LOOKME_ERR_INVALID_ARG, "top_k %d outside [1, min(n_prims, %d)]", top_k, LOOKME_MAX_TOP_K);
+    if (N > 0 && (!queries || !scene_out || !prim_out || !weight_out))
+        return fail(LOOKME_ERR_INVALID_ARG, "queries, scene_out, prim_out and weight_out are required");
+    if (N > 0 && !aligned16(queries)) return fail(LOOKME_ERR_INVALID_ARG, "queries must be 16-byte aligned");
+    if (t->n_loaded != d.n_scenes)
+        return fail(LOOKME_ERR_STATE, "%lld of %lld scenes loaded", (long long)t->n_loaded, (long long)d.n_scenes);
+    if (d.residency == LOOKME_RES_HOST_STAGED && std::min<int64_t>(N, d.n_scenes) > t->n_slots)
+        return fail(LOOKME_ERR_UNSUPPORTED, "up to %lld routed scenes but only %lld staging slots",
+                    (long long)std::min<int64_t>(N, d.n_scenes), (long long)t->n_slots);
+    if (N == 0) return LOOKME_OK;
+    DeviceGuard guard(d.device);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if ((st = ensure_scratch(t, N, s)) != LOOKME_OK) return st;
+    LaunchCtx ctx{s, t->num_sms};
+    const int dk = (int)d.d_key;
+    const float* bias = t->has_bias ? t->bias : nullptr;
+
+    st = launch(t, s, KID_PREP, [&] { return launch_prep(ctx, d.dtype, queries, N, dk, t->qnorm, qnorm_out, t->best); });
+    if (st != LOOKME_OK) return st;
+    if (t->tc_route) {
+        CUtensorMap mq;
+        if (!encode_bf16_2d(&mq, queries, N, dk, 128))
+            return fail(LOOKME_ERR_CUDA, "cuTensorMapEncodeTiled failed for the queries");
+        const void* mc[3] = {&t->tmap_c[0], &t->tmap_c[1], &t->tmap_c[2]};
+        st = launch(t, s, KID_ROUTE_TC, [&] {
+            return launch_route_tc(ctx, &mq, mc, N, d.n_scenes, dk, t->inv_cnorm, bias, t->qnorm, t->best, t->status);
+        });
+    } else {
+        st = launch(t, s, KID_ROUTE_SIMT, [&] {
+            return launch_route_simt(ctx, d.dtype, queries, t->cent, N, d.n_scenes, dk, t->inv_cnorm, bias, t->qnorm,
+                                     t->best);
+        });
+    }
+    if (st != LOOKME_OK) return st;
+    st = launch(t, s, KID_BUCKET, [&] {
+        return launch_bucket(ctx, t->best, N, d.n_scenes, scene_out, t->perm, t->work, t->routed, t->counters);
+    });
+    if (st != LOOKME_OK) return st;
+    const bool staged = d.residency == LOOKME_RES_HOST_STAGED;
+    if (staged) {
+        const int64_t block_bytes = d.n_prims * d.d_key * (int64_t)t->esz;
+        st = launch(t, s, KID_STAGE, [&] {
+            return launch_stage(ctx, t->keys, t->slots, block_bytes, t->n_slots, t->routed, t->counters);
+        });
+        if (st != LOOKME_OK) return st;
+    }
+    ScoreArgs a;
+    a.dtype = d.dtype;
+    a.q = queries;
+    a.keys = staged ? t->slots : t->keys;
+    a.P = d.n_prims;
+    a.dk = dk;
+    a.top_k = top_k;
+    a.scale = (float)(1.0 / std::sqrt((double)dk));
+    a.work = t->work;
+    a.n_work = t->counters;
+    a.perm = t->perm;
+    a.use_slots = staged ? 1 : 0;
+    a.prim_out = prim_out;
+    a.weight_out = weight_out;
+    a.status = t->status;
+    st = launch(t, s, KID_SCORE, [&] { return launch_score(ctx, a); });
+    if (st != LOOKME_OK) return st;
+    t->last_tokens = N;
+    return LOOKME_OK;
+}
+
+lookme_status lookme_inject(lookme_table* t, const int32_t* scene, const int32_t* prim, const float* weight,
+                            int64_t N, int32_t top_k, const float* priority, const int64_t* seg_offsets,
+                            int32_t n_seg, double keep_ratio, void* const* hidden, int32_t n_layers,
+                            uint8_t* mask_out, int32_t* sel_out, lookme_stream stream) {
+    lookme_status st = check_table(t);
+    if (st != LOOKME_OK) return st;
+    const lookme_table_desc& d = t->d;
+    if (N < 0 || N > INT32_MAX / 2) return fail(LOOKME_ERR_INVALID_ARG, "n_tokens %lld out of range", (long long)N);
+    if (top_k < 1 || top_k > LOOKME_MAX_TOP_K || top_k > d.n_prims)
+        return fail(LOOKME_ERR_INVALID_ARG, "top_k %d outside [1, min(n_prims, %d)]", top_k, LOOKME_MAX_TOP_K);
+    if (!(keep_ratio >= 0.0 && keep_ratio <= 1.0)) return fail(LOOKME_ERR_INVALID_ARG, "keep_ratio outside [0, 1]");
+    if (n_layers < 1 || n_layers > LOOKME_MAX_LAYERS)
+        return fail(LOOKME_ERR_INVALID_ARG, "n_layers %d outside [1, %d]", n_layers, LOOKME_MAX_LAYERS);
+    if (!hidden) return fail(LOOKME_ERR_INVALID_ARG, "hidden is NULL");
+    for (int l = 0; l < n_layers; ++l) {
+        if (N > 0 && (!hidden[l] || !aligned16(hidden[l])))
+            return fail(LOOKME_ERR_INVALID_ARG, "hidden[%d] is NULL or not 16-byte aligned", l);
+    }
+    std::vector<int64_t> off;
+    if (seg_offsets) {
+        if (n_seg < 1 || n_seg > LOOKME_MAX_SEGMENTS)
+            return fail(LOOKME_ERR_INVALID_ARG, "n_seg %d outside [1, %d]", n_seg, LOOKME_MAX_SEGMENTS);
+        off.assign(seg_offsets, seg_offsets + n_seg + 1);
+        if (off[0] != 0 || off[n_seg] != N)
+            return fail(LOOKME_ERR_INVALID_ARG, "seg_offsets must start at 0 and end at n_tokens");
+        for (int i = 0; i < n_seg; ++i)
+            if (off[i + 1] < off[i]) return fail(LOOKME_ERR_INVALID_ARG, "seg_offsets must be non-decreasing");
+    } else {
+        n_seg = 1;
+        off = {0, N};
+    }
+    if (N == 0) return LOOKME_OK;
+    if (!scene || !prim || !weight) return fail(LOOKME_ERR_INVALID_ARG, "scene, prim and weight are required");
+    if (!priority && t->last_tokens != N)
+        return fail(LOOKME_ERR_STATE, "default priority needs a lookup of %lld tokens first", (long long)N);
+    int64_t n_sel = 0;
+    for (int i = 0; i < n_seg; ++i) n_sel += (int64_t)std::floor((double)(off[i + 1] - off[i]) * keep_ratio);
+
+    DeviceGuard guard(d.device);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if ((st = ensure_scratch(t, N, s)) != LOOKME_OK) return st;
+    LaunchCtx ctx{s, t->num_sms};
+    uint8_t* mask = mask_out ? mask_out : t->mask;
+    int32_t* sel = sel_out ? sel_out : t->sel;
+    const float* pr = priority ? priority : t->qnorm;
+    st = launch(t, s, KID_SELECT, [&] { return launch_select(ctx, pr, N, off.data(), n_seg, keep_ratio, mask, sel); });
+    if (st != LOOKME_OK) return st;
+    if (n_sel == 0) return LOOKME_OK;
+    InjectArgs a;
+    a.dtype = d.dtype;
+    a.values = t->values;
+    a.P = d.n_prims;
+    a.dv = (int)d.d_value;
+    a.top_k = top_k;
+    a.scene = scene;
+    a.prim = prim;
+    a.weight = weight;
+    a.sel = sel;
+    a.n_sel = n_sel;
+    a.N = N;
+    a.S = d.n_scenes;
+    a.n_layers = n_layers;
+    for (int l = 0; l < n_layers; ++l) a.hidden[l] = hidden[l];
+    return launch(t, s, KID_INJECT, [&] { return launch_inject(ctx, a); });
+}
+
+lookme_status lookme_last_lookup_stats(lookme_table* t, lookme_lookup_stats* out, lookme_stream stream) {
+    lookme_status st = check_table(t);
+    if (st != LOOKME_OK) return st;
+    if (!out) return fail(LOOKME_ERR_INVALID_ARG, "out is NULL");
+    memset(out, 0, sizeof(*out));
+    if (t->last_tokens < 0 || !t->counters) return LOOKME_OK;
+    DeviceGuard guard(t->d.device);
+    int32_t c[4];
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemcpyAsync(c, t->counters, sizeof(c), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(t, e, "read lookup stats");
+    out->n_tokens = t->last_tokens;
+    out->n_work_items = c[0];
+    out->n_routed_scenes = c[1];
+    out->staged_bytes = t->d.residency == LOOKME_RES_HOST_STAGED
+                            ? (int64_t)c[1] * t->d.n_prims * t->d.d_key * (int64_t)t->esz
+                            : 0;
+    return LOOKME_OK;
+}
+
+lookme_status lookme_device_status(lookme_table* t, uint32_t* status, int reset, lookme_stream stream) {
+    if (!t || !status) return fail(LOOKME_ERR_INVALID_ARG, "NULL argument");
+    DeviceGuard guard(t->d.device);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemcpyAsync(status, t->status, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e == cudaSuccess && reset) e = cudaMemsetAsync(t->status, 0, sizeof(uint32_t), s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(t, e, "read device status");
+    return LOOKME_OK;
+}
+
+uint64_t lookme_launch_count(const lookme_table* t) { return t ? t->launches : 0; }
+
+lookme_status lookme_trace_enable(lookme_table* t, int enable) {
+    if (!t) return fail(LOOKME_ERR_INVALID_ARG, "table is NULL");
+    t->trace = enable != 0;
+    return LOOKME_OK;
+}
+
+lookme_status lookme_trace_read(lookme_table* t, lookme_trace_record* out, int32_t max, int32_t* n_out) {
+    if (!t || !n_out || (max > 0 && !out)) return fail(LOOKME_ERR_INVALID_ARG, "NULL argument");
+    DeviceGuard guard(t->d.device);
+    int32_t n = 0;
+    lookme_status st = LOOKME_OK;
+    for (auto& te : t->trace_log) {
+        float ms = 0.f;
+        cudaError_t e = cudaEventSynchronize(te.stop);
+        if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, te.start, te.stop);
+        if (e != cudaSuccess && st == LOOKME_OK) st = cuda_fail(t, e, "trace event");
+        if (n < max) out[n++] = lookme_trace_record{te.kernel, ms};
+        t->event_pool.push_back(te.start);
+        t->event_pool.push_back(te.stop);
+    }
+    t->trace_log.clear();
+    *n_out = n;
+    return st;
+}
+
+}  // extern "C"

@@ -54,6 +54,7 @@ def check_two_scene_example(o):
     assert r["scene"].tolist() == e["scene"], r["scene"]
     _close(r["gap1"], e["gap1"], what="gap1")
     _close(r["qnorm"], e["qnorm"], what="qnorm")
+    _close(o.query_norms(q), e["qnorm"], what="query_norms")
     p = o.primitives(q, r["scene"], np.array(x["keys"]), x["top_k"])
     assert p["prim"].tolist() == e["prim"], p["prim"]
     _close(p["logit"], e["logit"], what="logit")
