@@ -82,14 +82,31 @@ __global__ void __launch_bounds__(k5::kThreads, 1) k5_select(const __grid_consta
                 if ((k & pmask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1);
             }
             __syncthreads();
-            if (tid == 0) {
-                int above = 0, d = 255;
-                for (; d > 0; --d) {
-                    if (above + hist[d] >= remaining) break;
-                    above += hist[d];
+            // One warp finds the digit holding the r-th largest key: lane l
+            // owns bins 255 - 8 l ... 248 - 8 l (descending), an exclusive
+            // prefix over lanes gives the count above each lane's bins.
+            if (tid < 32) {
+                const int top = 255 - 8 * tid;
+                int local = 0;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) local += hist[top - i];
+                int inc = local;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int n = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+                    if (tid >= o) inc += n;
                 }
-                sh_prefix = prefix | ((uint32_t)d << shift);
-                sh_remaining = remaining - above;
+                const int excl = inc - local;
+                if (excl < remaining && remaining <= inc) {
+                    int above = excl, d = top;
+                    for (int i = 0; i < 8; ++i) {
+                        d = top - i;
+                        if (above + hist[d] >= remaining) break;
+                        above += hist[d];
+                    }
+                    sh_prefix = prefix | ((uint32_t)d << shift);
+                    sh_remaining = remaining - above;
+                }
             }
             __syncthreads();
             prefix = sh_prefix;
@@ -143,7 +160,7 @@ cudaError_t launch_select(const LaunchCtx& c, const float* priority, int64_t N, 
 
 // ---------------------------------------------------------------- K4 inject
 namespace k4 {
-constexpr int kThreads = 128;
+constexpr int kThreads = 256;
 
 struct Params {
     const void* values;
@@ -164,6 +181,7 @@ struct Params {
 template <typename T>
 __global__ void __launch_bounds__(k4::kThreads) k4_inject(const __grid_constant__ k4::Params p) {
     constexpr int EPC = Vec16<T>::N;
+    constexpr int BATCH = 8;  // value rows in flight per thread
     __shared__ const uint4* rows[LOOKME_MAX_TOP_K];
     __shared__ float w[LOOKME_MAX_TOP_K];
     const int64_t t = p.sel[blockIdx.x];
@@ -176,32 +194,31 @@ __global__ void __launch_bounds__(k4::kThreads) k4_inject(const __grid_constant_
     __syncthreads();
     const int chunks = p.dv / EPC;
     for (int ch = threadIdx.x; ch < chunks; ch += blockDim.x) {
+        uint4* h0 = reinterpret_cast<uint4*>(reinterpret_cast<T*>(p.hidden[0]) + t * p.dv) + ch;
+        const uint4 hv0 = *h0;  // issued together with the value rows
         float acc[EPC];
 #pragma unroll
         for (int e = 0; e < EPC; ++e) acc[e] = 0.f;
-        int j = 0;
-        for (; j + 4 <= p.top_k; j += 4) {
-            uint4 v[4];
+        for (int j0 = 0; j0 < p.top_k; j0 += BATCH) {
+            uint4 v[BATCH];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) v[u] = __ldg(rows[j + u] + ch);
+            for (int u = 0; u < BATCH; ++u)
+                if (j0 + u < p.top_k) v[u] = __ldg(rows[j0 + u] + ch);
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                float f[EPC];
-                Vec16<T>::unpack(v[u], f);
+            for (int u = 0; u < BATCH; ++u) {
+                if (j0 + u < p.top_k) {
+                    float f[EPC];
+                    Vec16<T>::unpack(v[u], f);
+                    const float wu = w[j0 + u];
 #pragma unroll
-                for (int e = 0; e < EPC; ++e) acc[e] = fmaf(w[j + u], f[e], acc[e]);
+                    for (int e = 0; e < EPC; ++e) acc[e] = fmaf(wu, f[e], acc[e]);
+                }
             }
-        }
-        for (; j < p.top_k; ++j) {
-            float f[EPC];
-            Vec16<T>::unpack(__ldg(rows[j] + ch), f);
-#pragma unroll
-            for (int e = 0; e < EPC; ++e) acc[e] = fmaf(w[j], f[e], acc[e]);
         }
         for (int l = 0; l < p.n_layers; ++l) {
             uint4* h = reinterpret_cast<uint4*>(reinterpret_cast<T*>(p.hidden[l]) + t * p.dv) + ch;
             float f[EPC];
-            Vec16<T>::unpack(*h, f);
+            Vec16<T>::unpack(l == 0 ? hv0 : *h, f);
 #pragma unroll
             for (int e = 0; e < EPC; ++e) f[e] += acc[e];
             *h = Vec16<T>::pack(f);
@@ -224,10 +241,14 @@ cudaError_t launch_inject(const LaunchCtx& c, const InjectArgs& a) {
     p.S = a.S;
     p.n_layers = a.n_layers;
     for (int l = 0; l < a.n_layers; ++l) p.hidden[l] = a.hidden[l];
+    // One 16-byte chunk of the row per thread where the row allows it.
+    const int chunks = a.dv / (a.dtype == LOOKME_BF16 ? 8 : 4);
+    int threads = (chunks + 31) / 32 * 32;
+    if (threads > k4::kThreads) threads = k4::kThreads;
     if (a.dtype == LOOKME_BF16)
-        k4_inject<__nv_bfloat16><<<(unsigned)a.n_sel, k4::kThreads, 0, c.stream>>>(p);
+        k4_inject<__nv_bfloat16><<<(unsigned)a.n_sel, threads, 0, c.stream>>>(p);
     else
-        k4_inject<float><<<(unsigned)a.n_sel, k4::kThreads, 0, c.stream>>>(p);
+        k4_inject<float><<<(unsigned)a.n_sel, threads, 0, c.stream>>>(p);
     return cudaGetLastError();
 }
 

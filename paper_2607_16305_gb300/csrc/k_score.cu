@@ -175,8 +175,8 @@ __global__ void __launch_bounds__(k3::kThreads, 2)
         if (warp < nb) {
             const float* z = zs + warp * P;
             uint64_t taken = 0ull;  // bit i: element lane + 32 i already selected
-            float my_z = 0.f;
-            int my_p = 0;
+            float my_z[2] = {0.f, 0.f};  // output slots lane and lane + 32
+            int my_p[2] = {0, 0};
             for (int kk = 0; kk < top_k; ++kk) {
                 float bz = 0.f;
                 int bp = -1;
@@ -200,20 +200,29 @@ __global__ void __launch_bounds__(k3::kThreads, 2)
                     }
                 }
                 if (bp >= 0 && (bp & 31) == lane) taken |= 1ull << (bp >> 5);
-                if (lane == kk) {
-                    my_z = bz;
-                    my_p = bp;
+                if ((kk & 31) == lane) {
+                    my_z[kk >> 5] = bz;
+                    my_p[kk >> 5] = bp;
                 }
             }
-            const float zmax = __shfl_sync(0xFFFFFFFFu, my_z, 0);
-            const float e = lane < top_k ? expf(my_z - zmax) : 0.f;
-            float sum = e;
+            const float zmax = __shfl_sync(0xFFFFFFFFu, my_z[0], 0);
+            float e[2];
+            float sum = 0.f;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                e[h] = (h * 32 + lane < top_k) ? expf(my_z[h] - zmax) : 0.f;
+                sum += e[h];
+            }
 #pragma unroll
             for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
-            if (lane < top_k) {
-                const int64_t t = perm[w.begin + warp];
-                prim_out[t * top_k + lane] = my_p;
-                weight_out[t * top_k + lane] = e / sum;
+            const int64_t t = perm[w.begin + warp];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int j = h * 32 + lane;
+                if (j < top_k) {
+                    prim_out[t * top_k + j] = my_p[h];
+                    weight_out[t * top_k + j] = e[h] / sum;
+                }
             }
         }
         __syncthreads();  // logits and queries are rewritten by the next item
