@@ -195,6 +195,29 @@ lookme_status lookme_trace_enable(lookme_table* table, int enable);
 lookme_status lookme_trace_read(lookme_table* table, lookme_trace_record* out, int32_t max, int32_t* n_out);
 const char* lookme_kernel_name(int32_t kernel);
 
+/* Level-1 routing only (scene_out[t] for every query, exactly as
+ * lookme_lookup's scene_out) without allocating anything.  The paper has no
+ * counterpart: this entry point exists for callers that cannot allocate
+ * device memory when they route, such as a serving loop whose device memory
+ * belongs to another allocator or a path that must avoid the device-wide
+ * synchronisation an allocation can cause.  Its per-token scratch lives in
+ * fixed device arrays built into the library, sized for
+ * LOOKME_ROUTE_STATIC_MAX_TOKENS tokens (768 KiB per device, held by every
+ * GPU that loads the library until the process exits).
+ *   queries    device [n_tokens][d_key], n_tokens <= LOOKME_ROUTE_STATIC_MAX_TOKENS
+ *              (larger requests fail with INVALID_ARG before anything runs)
+ *   scene_out  device [n_tokens] int32
+ * The first call on a device looks up the arrays' device addresses
+ * (cudaGetSymbolAddress) with that device current; make that first call
+ * before any stream capture.  All calls share the one scratch and each call
+ * re-initialises the part it uses, so calls that may overlap on the GPU (on
+ * different streams, or from different tables on the same device) race and
+ * must be serialised by the caller.
+ * Errors: INVALID_ARG, STATE (a scene not loaded yet), CUDA. */
+#define LOOKME_ROUTE_STATIC_MAX_TOKENS 65536
+lookme_status lookme_route_scenes_static(lookme_table* table, const void* queries, int64_t n_tokens,
+                                         int32_t* scene_out, lookme_stream stream);
+
 const char* lookme_status_string(lookme_status status);
 const char* lookme_last_error(void);
 

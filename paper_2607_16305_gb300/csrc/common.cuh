@@ -22,6 +22,7 @@ enum KernelId : int32_t {
     KID_STAGE = 7,       // K6: host -> HBM staging of routed key blocks
     KID_CENTROID = 8,    // load-time: centroid = mean of keys
     KID_CNORM = 9,       // load-time: 1 / ||centroid||
+    KID_ROUTE_DECODE = 10,  // argmax key -> scene id (allocation-free routing)
     KID_COUNT
 };
 

@@ -37,8 +37,8 @@ lookme_status fail(lookme_status st, const char* fmt, ...) {
     return st;
 }
 
-const char* kKernelNames[KID_COUNT] = {"prep", "route_tc", "route_simt", "bucket", "score",
-                                       "select", "inject", "stage", "centroid_mean", "inv_cnorm"};
+const char* kKernelNames[KID_COUNT] = {"prep",   "route_tc", "route_simt",    "bucket",    "score",       "select",
+                                       "inject", "stage",    "centroid_mean", "inv_cnorm", "route_decode"};
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point, so the
 // library does not link libcuda directly.
@@ -654,3 +654,105 @@ lookme_status lookme_trace_read(lookme_table* t, lookme_trace_record* out, int32
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Level-1 routing that allocates nothing.
+//
+// Some callers cannot allocate device memory at the point where they route
+// tokens: a serving loop whose device memory is owned by another allocator
+// (for example a framework's caching allocator holding the whole card), code
+// that must not pay the implicit device-wide synchronisation cudaMalloc and
+// cudaFree can cause, or a real-time path with a fixed memory budget.
+// lookme_route_scenes_static serves them: its per-token scratch (the packed
+// argmax keys and the query norms) lives in the two fixed arrays below, which
+// every GPU that loads this library holds until the process exits
+// (LOOKME_ROUTE_STATIC_MAX_TOKENS x 12 bytes = 768 KiB per device).  Host code
+// must not use the array names as device addresses: it asks the runtime for
+// them once per device with cudaGetSymbolAddress.
+static __device__ __align__(256) unsigned long long g_static_best[LOOKME_ROUTE_STATIC_MAX_TOKENS];
+static __device__ __align__(256) float g_static_qnorm[LOOKME_ROUTE_STATIC_MAX_TOKENS];
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+
+struct StaticScratch {
+    unsigned long long* best = nullptr;
+    float* qnorm = nullptr;
+};
+
+std::mutex g_static_mu;
+StaticScratch g_static_scratch[kMaxDevices];
+
+// Device addresses of the fixed arrays on `device`, which must be current.
+// Looked up on the first call per device and cached.
+lookme_status static_scratch(int device, StaticScratch* out) {
+    if (device < 0 || device >= kMaxDevices) return fail(LOOKME_ERR_UNSUPPORTED, "device %d out of range", device);
+    std::lock_guard<std::mutex> lock(g_static_mu);
+    StaticScratch& sc = g_static_scratch[device];
+    if (!sc.best) {
+        void* pb = nullptr;
+        void* pq = nullptr;
+        cudaError_t e = cudaGetSymbolAddress(&pb, g_static_best);
+        if (e != cudaSuccess) return fail(LOOKME_ERR_CUDA, "cudaGetSymbolAddress(best): %s", cudaGetErrorString(e));
+        e = cudaGetSymbolAddress(&pq, g_static_qnorm);
+        if (e != cudaSuccess) return fail(LOOKME_ERR_CUDA, "cudaGetSymbolAddress(qnorm): %s", cudaGetErrorString(e));
+        sc.best = static_cast<unsigned long long*>(pb);
+        sc.qnorm = static_cast<float*>(pq);
+    }
+    *out = sc;
+    return LOOKME_OK;
+}
+
+__global__ void k_route_static_decode(const unsigned long long* __restrict__ best, int64_t N, int64_t S,
+                                      int32_t* __restrict__ scene_out) {
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (t < N) scene_out[t] = unpack_scene(best[t], S);
+}
+
+}  // namespace
+
+extern "C" lookme_status lookme_route_scenes_static(lookme_table* t, const void* queries, int64_t N,
+                                                    int32_t* scene_out, lookme_stream stream) {
+    lookme_status st = check_table(t);
+    if (st != LOOKME_OK) return st;
+    const lookme_table_desc& d = t->d;
+    if (N < 0 || N > LOOKME_ROUTE_STATIC_MAX_TOKENS)
+        return fail(LOOKME_ERR_INVALID_ARG, "n_tokens %lld outside [0, %d], the size of the fixed scratch",
+                    (long long)N, LOOKME_ROUTE_STATIC_MAX_TOKENS);
+    if (N > 0 && (!queries || !scene_out)) return fail(LOOKME_ERR_INVALID_ARG, "queries and scene_out are required");
+    if (N > 0 && !aligned16(queries)) return fail(LOOKME_ERR_INVALID_ARG, "queries must be 16-byte aligned");
+    if (t->n_loaded != d.n_scenes)
+        return fail(LOOKME_ERR_STATE, "%lld of %lld scenes loaded", (long long)t->n_loaded, (long long)d.n_scenes);
+    if (N == 0) return LOOKME_OK;
+    DeviceGuard guard(d.device);
+    StaticScratch sc;
+    if ((st = static_scratch(d.device, &sc)) != LOOKME_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    LaunchCtx ctx{s, t->num_sms};
+    const int dk = (int)d.d_key;
+    const float* bias = t->has_bias ? t->bias : nullptr;
+    // The prep kernel rewrites every key the routing kernel reduces into, so
+    // leftovers of an earlier call never leak into this one.
+    st = launch(t, s, KID_PREP, [&] { return launch_prep(ctx, d.dtype, queries, N, dk, sc.qnorm, nullptr, sc.best); });
+    if (st != LOOKME_OK) return st;
+    if (t->tc_route) {
+        CUtensorMap mq;
+        if (!encode_bf16_2d(&mq, queries, N, dk, 128))
+            return fail(LOOKME_ERR_CUDA, "cuTensorMapEncodeTiled failed for the queries");
+        const void* mc[3] = {&t->tmap_c[0], &t->tmap_c[1], &t->tmap_c[2]};
+        st = launch(t, s, KID_ROUTE_TC, [&] {
+            return launch_route_tc(ctx, &mq, mc, N, d.n_scenes, dk, t->inv_cnorm, bias, sc.qnorm, sc.best, t->status);
+        });
+    } else {
+        st = launch(t, s, KID_ROUTE_SIMT, [&] {
+            return launch_route_simt(ctx, d.dtype, queries, t->cent, N, d.n_scenes, dk, t->inv_cnorm, bias, sc.qnorm,
+                                     sc.best);
+        });
+    }
+    if (st != LOOKME_OK) return st;
+    return launch(t, s, KID_ROUTE_DECODE, [&] {
+        k_route_static_decode<<<(unsigned)((N + 255) / 256), 256, 0, s>>>(sc.best, N, d.n_scenes, scene_out);
+        return cudaGetLastError();
+    });
+}

@@ -20,12 +20,13 @@ OK, ERR_INVALID_ARG, ERR_CUDA, ERR_OOM, ERR_TIMEOUT, ERR_STATE, ERR_UNSUPPORTED 
 BF16, FP32 = 0, 1
 RES_DEVICE, RES_HOST_STAGED = 0, 1
 MAX_TOP_K, MAX_LAYERS, MAX_SEGMENTS = 64, 64, 1024
+ROUTE_STATIC_MAX_TOKENS = 65536
 
 EXPORTS = [
     "lookme_table_create", "lookme_table_destroy", "lookme_load_scenes", "lookme_lookup", "lookme_inject",
     "lookme_reserve", "lookme_last_lookup_stats", "lookme_device_status", "lookme_launch_count",
     "lookme_trace_enable", "lookme_trace_read", "lookme_kernel_name", "lookme_status_string",
-    "lookme_last_error",
+    "lookme_last_error", "lookme_route_scenes_static",
 ]
 
 
@@ -80,6 +81,7 @@ def load(path: str = LIB_PATH):
         "lookme_kernel_name": ([I32], ctypes.c_char_p),
         "lookme_status_string": ([I32], ctypes.c_char_p),
         "lookme_last_error": ([], ctypes.c_char_p),
+        "lookme_route_scenes_static": ([P, P, I64, P, P], I32),
     }
     for name, (argtypes, restype) in sig.items():
         fn = getattr(lib, name)
