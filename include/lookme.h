@@ -90,7 +90,7 @@ typedef struct lookme_table lookme_table; /* opaque, owned by the library */
 #define LOOKME_MAX_SEGMENTS 1024   /* token-selection segments per inject call */
 #define LOOKME_MAX_SCENES 49152    /* n_scenes (bucketing keeps one counter per scene on chip) */
 #define LOOKME_MAX_PRIMS 2048      /* n_prims (level-2 keeps one logit per primitive on chip) */
-#define LOOKME_MAX_DKEY 2048       /* d_key */
+#define LOOKME_MAX_DKEY 1024       /* d_key */
 
 /* Create a table on desc->device.  Allocates the table storage (HBM, or
  * pinned host for HOST_STAGED), the centroids and, if desc->max_tokens > 0,

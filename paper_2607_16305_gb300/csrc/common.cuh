@@ -125,7 +125,7 @@ struct ScoreArgs {
     int top_k;
     float scale;          // 1 / sqrt(d_k)
     const WorkItem* work;
-    const int32_t* n_work;
+    int32_t* counters;    // [0] work items (from bucketing), [3] work-taking counter (reset by bucketing)
     const int32_t* perm;
     int use_slots;        // index key blocks by WorkItem::slot instead of ::scene
     int32_t* prim_out;
@@ -133,6 +133,8 @@ struct ScoreArgs {
     uint32_t* status;
 };
 cudaError_t launch_score(const LaunchCtx& c, const ScoreArgs& a);
+// Whether the level-2 kernel's shared-memory plan fits this table shape.
+bool score_shape_supported(int dtype, int64_t P, int dk);
 // K5
 cudaError_t launch_select(const LaunchCtx& c, const float* priority, int64_t N, const int64_t* seg_off_host,
                           int n_seg, double keep_ratio, uint8_t* mask, int32_t* sel);

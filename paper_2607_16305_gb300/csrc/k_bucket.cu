@@ -10,7 +10,8 @@
 //                  scene order: every scene's bucket cut into chunks
 //   routed         the distinct routed scenes in increasing order; a scene's
 //                  position in it is its `slot`
-//   counters[0..2] number of work items, of routed scenes, largest bucket
+//   counters[0..3] number of work items, of routed scenes, largest bucket;
+//                  [3] is reset to 0 for the level-2 kernel's work taking
 #include "common.cuh"
 
 namespace lookme {
@@ -116,6 +117,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         counters[0] = total.y;
         counters[1] = total.z;
         counters[2] = max_bucket;
+        counters[3] = 0;  // level-2 work-taking counter
     }
     for (int64_t t = tid; t < N; t += kThreads) {
         const int32_t s = unpack_scene(best[t], S);

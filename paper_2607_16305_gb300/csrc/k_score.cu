@@ -5,37 +5,58 @@
 //   w_t  = softmax over z_t[I_t]
 //
 // The path is HBM-bound: a scene's key block (N_p x d_k) is read once per
-// work item while a bucket holds only a few tokens.  Each CTA walks a static
-// share of the work list; one thread streams the key blocks into a ring of
-// shared-memory stages with cp.async.bulk (completion on mbarriers) and runs
-// ahead across work items, so the next item's keys are in flight while the
-// current item finishes its top-k.  Threads own key rows (TPR threads per
-// row, 8 x 16-byte chunks each), read their chunks in a lane-rotated order so
-// that eight consecutive lanes hit eight different bank groups, dot them with
-// the (broadcast) fp32 queries of the item's tokens, and reduce across the
-// TPR lanes with shuffles.  Logits land in shared memory; one warp per token
-// then extracts the top-k and the softmax weights.
+// work item while a bucket holds only a few tokens, so the kernel keeps many
+// bytes in flight and keeps dependent global reads and the top-k off the
+// warps that consume the key stream.  One CTA per SM, three warp roles:
+//   producer warp    takes work items from a global counter, reads the item's
+//                    token ids, bulk-copies (cp.async.bulk) their query rows
+//                    into an item slot and streams the scene's key block
+//                    through a ring of 32 KiB stages; every copy completes on
+//                    an mbarrier
+//   8 compute warps  convert the item's queries to fp32, dot each key row
+//                    with them (threads own key rows: TPR threads per row, 8 x
+//                    16-byte chunks each, read in a lane-rotated order so
+//                    eight consecutive lanes hit eight bank groups; the token
+//                    loop is specialised on the bucket size), reduce across
+//                    the row's threads with shuffles and write the logits
+//                    into one of two logit buffers
+//   4 top-k warps    one token per warp: top-k by repeated warp argmax
+//                    (redux.sync on order-preserving keys, ties to the lower
+//                    primitive), softmax, outputs; they run on buffer i while
+//                    the compute warps fill buffer i+1
+// Compute warps synchronise among themselves with a named barrier whose OR
+// reduction makes the abort decision uniform; every wait is bounded.
 #include "common.cuh"
 #include "sm100.cuh"
 
 namespace lookme {
 
 namespace k3 {
-constexpr int kThreads = 256;
-constexpr int kTok = kTokensPerItem;  // tokens per work item == warps per CTA
-constexpr int kStages = 3;
+constexpr int kComputeWarps = 8;
+constexpr int kCompute = kComputeWarps * 32;
+constexpr int kTopkWarps = 4;
+constexpr int kProducerWarp = kComputeWarps + kTopkWarps;
+constexpr int kThreads = (kProducerWarp + 1) * 32;
+constexpr int kTok = kTokensPerItem;
+constexpr int kMaxItemSlots = 4;
+constexpr int kMaxZBufs = 2;
 constexpr int kStageBytes = 32768;
+constexpr int kMaxStages = 6;
 constexpr uint64_t kTimeoutNs = 1000000000ull;
+constexpr int kSmemLimit = 227 * 1024;
 
 struct Geometry {
-    int row_bytes;       // d_k * element size
-    int row_chunks;      // 16-byte chunks per key row
-    int tpr;             // threads per key row (power of two)
-    int rows_per_stage;  // key rows per ring stage
-    int stages_per_item; // ring stages per work item (covers N_p rows)
-    int q_floats;        // floats of the per-item query buffer
-    int z_floats;        // floats of the per-item logit buffer
-    int smem;            // dynamic shared memory bytes
+    int row_bytes;        // d_k * element size
+    int row_chunks;       // 16-byte chunks per key row
+    int tpr;              // threads per key row (power of two)
+    int rows_per_stage;   // key rows per ring stage
+    int stages_per_item;  // ring stages per work item (covers N_p rows)
+    int n_stages;         // ring depth
+    int n_items;          // item slots (query rows + token ids)
+    int n_z;              // logit buffers
+    int qraw_bytes;       // one item slot of raw query rows
+    int off_qraw, off_qf, off_z, off_bar, off_items;
+    int smem;
 };
 
 inline Geometry geometry(int dtype, int64_t P, int dk) {
@@ -46,207 +67,346 @@ inline Geometry geometry(int dtype, int64_t P, int dk) {
     const int need = (g.row_chunks + 7) / 8;
     g.tpr = 1;
     while (g.tpr < need) g.tpr <<= 1;
-    g.rows_per_stage = kThreads / g.tpr;
+    g.rows_per_stage = kCompute / g.tpr;
     g.stages_per_item = (int)((P + g.rows_per_stage - 1) / g.rows_per_stage);
-    g.q_floats = kTok * dk;
-    g.z_floats = kTok * (int)P;
-    g.smem = kStages * kStageBytes + (g.q_floats + g.z_floats) * 4 + kStages * 8 + 16;
+    g.qraw_bytes = (kTok * g.row_bytes + 127) / 128 * 128;
+    const int zbytes = kTok * (int)P * 4;
+    // Deepest ring first; give up logit and item buffering only if the ring would be too shallow.
+    const int plans[3][2] = {{kMaxItemSlots, kMaxZBufs}, {kMaxItemSlots, 1}, {2, 1}};
+    for (int i = 0; i < 3; ++i) {
+        g.n_items = plans[i][0];
+        g.n_z = plans[i][1];
+        const int fixed = g.n_items * g.qraw_bytes + kTok * dk * 4 + g.n_z * zbytes + 1024;
+        g.n_stages = (kSmemLimit - fixed) / kStageBytes;
+        if (g.n_stages > kMaxStages) g.n_stages = kMaxStages;
+        if (g.n_stages >= 3) break;
+    }
+    g.off_qraw = g.n_stages * kStageBytes;
+    g.off_qf = g.off_qraw + g.n_items * g.qraw_bytes;
+    g.off_z = g.off_qf + kTok * dk * 4;
+    g.off_bar = (g.off_z + g.n_z * zbytes + 7) / 8 * 8;
+    g.off_items = g.off_bar + (2 * kMaxStages + 2 * kMaxItemSlots + 2 * kMaxZBufs) * 8;
+    g.smem = g.off_items + kMaxItemSlots * ((int)sizeof(WorkItem) + kTok * 4) + 16;
     return g;
+}
+
+// Named barrier 1 over the compute warps, returning the OR of `v` over them.
+__device__ __forceinline__ bool compute_sync_or(bool v) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.or.pred q, 1, %2, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"((uint32_t)v), "n"(kCompute)
+        : "memory");
+    return r != 0;
+}
+
+// One ring stage: the logits of this thread's key row for the item's NB tokens.
+template <typename T, int NB>
+__device__ __forceinline__ void score_stage(const uint8_t* krow, const float* qf, const Geometry& g, int seg, int lane,
+                                            int64_t row, int64_t P, float scale, float* zs) {
+    constexpr int EPC = Vec16<T>::N;
+    constexpr int H = EPC / 4;
+    float a0[NB], a1[NB];
+#pragma unroll
+    for (int j = 0; j < NB; ++j) a0[j] = a1[j] = 0.f;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+        const int ch = seg * 8 + ((c + lane) & 7);
+        if (ch < g.row_chunks) {
+            float kf[EPC];
+            Vec16<T>::unpack(*reinterpret_cast<const uint4*>(krow + ch * 16), kf);
+#pragma unroll
+            for (int j = 0; j < NB; ++j) {
+#pragma unroll
+                for (int h = 0; h < H; ++h) {
+                    const float4 qv = *reinterpret_cast<const float4*>(qf + ((j * H + h) * g.row_chunks + ch) * 4);
+                    a0[j] = fmaf(kf[h * 4 + 0], qv.x, a0[j]);
+                    a1[j] = fmaf(kf[h * 4 + 1], qv.y, a1[j]);
+                    a0[j] = fmaf(kf[h * 4 + 2], qv.z, a0[j]);
+                    a1[j] = fmaf(kf[h * 4 + 3], qv.w, a1[j]);
+                }
+            }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < NB; ++j) {
+        float acc = a0[j] + a1[j];
+        for (int o = g.tpr / 2; o; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
+        if (seg == 0 && row < P) zs[j * P + row] = acc * scale;
+    }
+}
+
+// Inverse of orderable(): the float whose order key is u.
+__device__ __forceinline__ float from_orderable(uint32_t u) {
+    return __uint_as_float((u & 0x80000000u) ? (u & 0x7FFFFFFFu) : ~u);
+}
+
+// Top-k of z[0..P) by one warp (larger z first, lower index on ties) and the
+// softmax over the selected logits; writes prim/weight of token t.
+__device__ __forceinline__ void topk_token(const float* z, int64_t P, int top_k, int lane, int64_t t,
+                                           int32_t* prim_out, float* weight_out) {
+    // Each lane keeps the best untaken element of its slice p = lane + 32 i.
+    uint64_t taken = 0ull;
+    auto local_best = [&](uint32_t& key, uint32_t& pb) {
+        key = 0u;
+        pb = 0xFFFFFFFFu;
+        int i = 0;
+        for (int64_t p = lane; p < P; p += 32, ++i) {
+            if (!((taken >> i) & 1ull)) {
+                const uint32_t k = orderable(z[p]);
+                if (pb == 0xFFFFFFFFu || k > key) {
+                    key = k;
+                    pb = (uint32_t)p;
+                }
+            }
+        }
+    };
+    uint32_t key, pb;
+    local_best(key, pb);
+    float my_z[2] = {0.f, 0.f};  // output slots lane and lane + 32
+    int my_p[2] = {0, 0};
+    for (int kk = 0; kk < top_k; ++kk) {
+        const uint32_t kmax = __reduce_max_sync(0xFFFFFFFFu, pb == 0xFFFFFFFFu ? 0u : key);
+        const uint32_t pmin = __reduce_min_sync(0xFFFFFFFFu, (pb != 0xFFFFFFFFu && key == kmax) ? pb : 0xFFFFFFFFu);
+        if ((kk & 31) == lane) {
+            if (kk < 32) {
+                my_z[0] = from_orderable(kmax);
+                my_p[0] = (int)pmin;
+            } else {
+                my_z[1] = from_orderable(kmax);
+                my_p[1] = (int)pmin;
+            }
+        }
+        if (pmin != 0xFFFFFFFFu && (int)(pmin & 31u) == lane) {
+            taken |= 1ull << (pmin >> 5);
+            local_best(key, pb);
+        }
+    }
+    const float zmax = __shfl_sync(0xFFFFFFFFu, my_z[0], 0);
+    float e[2];
+    float sum = 0.f;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        e[h] = (h * 32 + lane < top_k) ? expf(my_z[h] - zmax) : 0.f;
+        sum += e[h];
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int j = h * 32 + lane;
+        if (j < top_k) {
+            prim_out[t * top_k + j] = my_p[h];
+            weight_out[t * top_k + j] = e[h] / sum;
+        }
+    }
 }
 }  // namespace k3
 
 template <typename T>
-__global__ void __launch_bounds__(k3::kThreads, 2)
+__global__ void __launch_bounds__(k3::kThreads, 1)
     k3_score(const T* __restrict__ q, const T* __restrict__ keys, int64_t P, int dk, int top_k, float scale,
-             const WorkItem* __restrict__ work, const int32_t* __restrict__ n_work_ptr,
-             const int32_t* __restrict__ perm, int use_slots, int32_t* __restrict__ prim_out,
-             float* __restrict__ weight_out, uint32_t* __restrict__ status, k3::Geometry g) {
+             const WorkItem* __restrict__ work, int32_t* __restrict__ counters, const int32_t* __restrict__ perm,
+             int use_slots, int32_t* __restrict__ prim_out, float* __restrict__ weight_out,
+             uint32_t* __restrict__ status, const __grid_constant__ k3::Geometry g) {
     using namespace k3;
-    constexpr int EPC = Vec16<T>::N;   // elements per 16-byte chunk
-    constexpr int H = EPC / 4;         // 16-byte halves of a chunk's fp32 query values
+    constexpr int EPC = Vec16<T>::N;
+    constexpr int H = EPC / 4;
     extern __shared__ __align__(128) uint8_t smem[];
     uint8_t* ring = smem;
-    float* qs = reinterpret_cast<float*>(ring + kStages * kStageBytes);
-    float* zs = qs + g.q_floats;
-    uint64_t* full = reinterpret_cast<uint64_t*>(zs + g.z_floats);
-    volatile int* abort = reinterpret_cast<volatile int*>(full + kStages);
+    uint8_t* qraw = smem + g.off_qraw;
+    float* qf = reinterpret_cast<float*>(smem + g.off_qf);
+    float* zbase = reinterpret_cast<float*>(smem + g.off_z);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + g.off_bar);
+    uint64_t* empty = full + kMaxStages;
+    uint64_t* ifull = empty + kMaxStages;
+    uint64_t* iempty = ifull + kMaxItemSlots;
+    uint64_t* zready = iempty + kMaxItemSlots;
+    uint64_t* zfree = zready + kMaxZBufs;
+    WorkItem* items = reinterpret_cast<WorkItem*>(smem + g.off_items);
+    int32_t* toks = reinterpret_cast<int32_t*>(items + kMaxItemSlots);
+    volatile int* abort = reinterpret_cast<volatile int*>(toks + kMaxItemSlots * kTok);
 
     const int tid = threadIdx.x, lane = tid % 32, warp = tid / 32;
-    const int n_work = *n_work_ptr;
-    const int G = gridDim.x;
-    const int my_items = n_work > (int)blockIdx.x ? (n_work - (int)blockIdx.x + G - 1) / G : 0;
-    if (my_items == 0) return;
-    const int64_t total_stages = (int64_t)my_items * g.stages_per_item;
+    const int n_work = counters[0];
+    const int64_t zstride = (int64_t)kTok * P;
 
     if (tid == 0) {
-        for (int i = 0; i < kStages; ++i) ptx::mbar_init(&full[i], 1);
+        for (int i = 0; i < g.n_stages; ++i) {
+            ptx::mbar_init(&full[i], 1);
+            ptx::mbar_init(&empty[i], kComputeWarps);
+        }
+        for (int i = 0; i < g.n_items; ++i) {
+            ptx::mbar_init(&ifull[i], 1);
+            ptx::mbar_init(&iempty[i], kTopkWarps);
+        }
+        for (int i = 0; i < g.n_z; ++i) {
+            ptx::mbar_init(&zready[i], kComputeWarps);
+            ptx::mbar_init(&zfree[i], kTopkWarps);
+        }
         *abort = 0;
         ptx::fence_mbar_init();
     }
     __syncthreads();
 
-    // Producer: ring stage `gs` (counted over this CTA's whole item sequence).
-    auto issue = [&](int64_t gs) {
-        const int it = (int)(gs / g.stages_per_item);
-        const int st = (int)(gs % g.stages_per_item);
-        const WorkItem w = work[blockIdx.x + (int64_t)it * G];
-        const int64_t block = use_slots ? w.slot : w.scene;
-        const int64_t row0 = (int64_t)st * g.rows_per_stage;
-        const int64_t rows = min((int64_t)g.rows_per_stage, P - row0);
-        const uint32_t bytes = (uint32_t)(rows * g.row_bytes);
-        const int slot = (int)(gs % kStages);
-        ptx::mbar_arrive_expect_tx(&full[slot], bytes);
-        const uint8_t* src = reinterpret_cast<const uint8_t*>(keys) + (block * P + row0) * (int64_t)g.row_bytes;
-        ptx::bulk_g2s(ring + slot * kStageBytes, src, bytes, &full[slot]);
-    };
-    if (tid == 0)
-        for (int64_t gs = 0; gs < total_stages && gs < kStages; ++gs) issue(gs);
-
-    const int r_in_stage = tid / g.tpr;
-    const int seg = tid % g.tpr;
-    int64_t gs = 0;
-    bool ok = true;
-    for (int it = 0; it < my_items && ok; ++it) {
-        const WorkItem w = work[blockIdx.x + (int64_t)it * G];
-        const int nb = w.count;
-        // Queries of the item's tokens -> fp32, layout [token][half][chunk][4].
-        for (int i = tid; i < nb * dk; i += kThreads) {
-            const int j = i / dk, e = i % dk;
-            const int32_t t = perm[w.begin + j];
-            const int ch = e / EPC, h = (e % EPC) / 4;
-            qs[((j * H + h) * g.row_chunks + ch) * 4 + (e & 3)] = to_f32(q[(int64_t)t * dk + e]);
-        }
-        __syncthreads();
-
-        for (int st = 0; st < g.stages_per_item; ++st, ++gs) {
-            const int slot = (int)(gs % kStages);
-            if (!ptx::mbar_wait(&full[slot], (uint32_t)((gs / kStages) & 1), abort, kTimeoutNs)) {
-                ok = false;
-            }
-            __syncthreads();
-            if (*abort) {
-                ok = false;
+    if (warp == kProducerWarp) {
+        // ------------------------------------------------------------ producer
+        uint32_t item_seq = 0;
+        int64_t stage_seq = 0;
+        bool ok = true;
+        for (;;) {
+            int wi = 0;
+            if (lane == 0) wi = atomicAdd(counters + 3, 1);
+            wi = __shfl_sync(0xFFFFFFFFu, wi, 0);
+            const int islot = (int)(item_seq % g.n_items);
+            const uint32_t ipar = (item_seq / g.n_items) & 1u;
+            if (lane == 0) ok = ptx::mbar_wait(&iempty[islot], ipar ^ 1u, abort, kTimeoutNs);
+            if (!__shfl_sync(0xFFFFFFFFu, (int)ok, 0)) break;
+            if (wi >= n_work) {
+                if (lane == 0) {
+                    items[islot].count = -1;  // end of work
+                    ptx::mbar_arrive(&ifull[islot]);
+                }
                 break;
             }
-            const uint8_t* krow = ring + slot * kStageBytes + r_in_stage * g.row_bytes;
-            float acc[kTok];
-#pragma unroll
-            for (int j = 0; j < kTok; ++j) acc[j] = 0.f;
-#pragma unroll
-            for (int c = 0; c < 8; ++c) {
-                const int ch = seg * 8 + ((c + lane) & 7);
-                if (ch < g.row_chunks) {
-                    float kf[EPC];
-                    Vec16<T>::unpack(*reinterpret_cast<const uint4*>(krow + ch * 16), kf);
-#pragma unroll
-                    for (int j = 0; j < kTok; ++j) {
-                        if (j < nb) {
-#pragma unroll
-                            for (int h = 0; h < H; ++h) {
-                                const float4 qv =
-                                    *reinterpret_cast<const float4*>(qs + ((j * H + h) * g.row_chunks + ch) * 4);
-                                acc[j] = fmaf(kf[h * 4 + 0], qv.x, acc[j]);
-                                acc[j] = fmaf(kf[h * 4 + 1], qv.y, acc[j]);
-                                acc[j] = fmaf(kf[h * 4 + 2], qv.z, acc[j]);
-                                acc[j] = fmaf(kf[h * 4 + 3], qv.w, acc[j]);
-                            }
-                        }
+            const WorkItem w = work[wi];
+            int32_t t = 0;
+            if (lane < w.count) {
+                t = perm[w.begin + lane];
+                toks[islot * kTok + lane] = t;
+            }
+            if (lane == 0) {
+                items[islot] = w;
+                ptx::mbar_arrive_expect_tx(&ifull[islot], (uint32_t)(w.count * g.row_bytes));
+            }
+            __syncwarp();
+            if (lane < w.count)
+                ptx::bulk_g2s(qraw + islot * g.qraw_bytes + lane * g.row_bytes,
+                              reinterpret_cast<const uint8_t*>(q) + (int64_t)t * g.row_bytes, (uint32_t)g.row_bytes,
+                              &ifull[islot]);
+            const int64_t block = use_slots ? w.slot : w.scene;
+            const uint8_t* src = reinterpret_cast<const uint8_t*>(keys) + block * P * (int64_t)g.row_bytes;
+            for (int st = 0; st < g.stages_per_item; ++st, ++stage_seq) {
+                const int slot = (int)(stage_seq % g.n_stages);
+                const uint32_t par = (uint32_t)((stage_seq / g.n_stages) & 1);
+                if (lane == 0) {
+                    ok = ptx::mbar_wait(&empty[slot], par ^ 1u, abort, kTimeoutNs);
+                    if (ok) {
+                        const int64_t row0 = (int64_t)st * g.rows_per_stage;
+                        const int64_t rows = min((int64_t)g.rows_per_stage, P - row0);
+                        const uint32_t bytes = (uint32_t)(rows * g.row_bytes);
+                        ptx::mbar_arrive_expect_tx(&full[slot], bytes);
+                        ptx::bulk_g2s(ring + slot * kStageBytes, src + row0 * g.row_bytes, bytes, &full[slot]);
                     }
                 }
+                if (!__shfl_sync(0xFFFFFFFFu, (int)ok, 0)) break;
             }
-#pragma unroll
-            for (int j = 0; j < kTok; ++j) {
-                if (j < nb) {
-                    for (int o = g.tpr / 2; o; o >>= 1) acc[j] += __shfl_xor_sync(0xFFFFFFFFu, acc[j], o);
-                }
-            }
-            const int64_t row = (int64_t)st * g.rows_per_stage + r_in_stage;
-            if (seg == 0 && row < P) {
-#pragma unroll
-                for (int j = 0; j < kTok; ++j)
-                    if (j < nb) zs[j * P + row] = acc[j] * scale;
-            }
-            __syncthreads();  // the slot is free and the logits are visible
-            if (tid == 0 && gs + kStages < total_stages) issue(gs + kStages);
+            if (!ok) break;
+            ++item_seq;
         }
-        if (!ok) break;
+        if (!ok && lane == 0) {
+            // Let the copies still in flight land before the CTA can exit.
+            for (int64_t s = stage_seq - g.n_stages; s < stage_seq; ++s)
+                if (s >= 0) ptx::mbar_wait_drain(&full[s % g.n_stages], (uint32_t)((s / g.n_stages) & 1), kTimeoutNs);
+            for (uint32_t s = item_seq >= (uint32_t)g.n_items ? item_seq - g.n_items + 1 : 0; s <= item_seq; ++s)
+                ptx::mbar_wait_drain(&ifull[s % g.n_items], (s / g.n_items) & 1u, kTimeoutNs);
+            atomicOr(status, STATUS_WAIT_TIMEOUT);
+        }
+        return;
+    }
 
-        // Top-k and softmax: warp j handles token j of the item.
-        if (warp < nb) {
-            const float* z = zs + warp * P;
-            uint64_t taken = 0ull;  // bit i: element lane + 32 i already selected
-            float my_z[2] = {0.f, 0.f};  // output slots lane and lane + 32
-            int my_p[2] = {0, 0};
-            for (int kk = 0; kk < top_k; ++kk) {
-                float bz = 0.f;
-                int bp = -1;
-                int i = 0;
-                for (int64_t p = lane; p < P; p += 32, ++i) {
-                    if (!((taken >> i) & 1ull)) {
-                        const float zz = z[p];
-                        if (bp < 0 || zz > bz) {
-                            bz = zz;
-                            bp = (int)p;
-                        }
-                    }
-                }
-#pragma unroll
-                for (int o = 16; o; o >>= 1) {
-                    const float oz = __shfl_xor_sync(0xFFFFFFFFu, bz, o);
-                    const int op = __shfl_xor_sync(0xFFFFFFFFu, bp, o);
-                    if (op >= 0 && (bp < 0 || oz > bz || (oz == bz && op < bp))) {
-                        bz = oz;
-                        bp = op;
-                    }
-                }
-                if (bp >= 0 && (bp & 31) == lane) taken |= 1ull << (bp >> 5);
-                if ((kk & 31) == lane) {
-                    my_z[kk >> 5] = bz;
-                    my_p[kk >> 5] = bp;
-                }
-            }
-            const float zmax = __shfl_sync(0xFFFFFFFFu, my_z[0], 0);
-            float e[2];
-            float sum = 0.f;
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                e[h] = (h * 32 + lane < top_k) ? expf(my_z[h] - zmax) : 0.f;
-                sum += e[h];
-            }
-#pragma unroll
-            for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
-            const int64_t t = perm[w.begin + warp];
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int j = h * 32 + lane;
-                if (j < top_k) {
-                    prim_out[t * top_k + j] = my_p[h];
-                    weight_out[t * top_k + j] = e[h] / sum;
-                }
+    if (warp >= kComputeWarps) {
+        // ------------------------------------------------------- top-k warps
+        const int tw = warp - kComputeWarps;
+        for (uint32_t item_seq = 0;; ++item_seq) {
+            const int islot = (int)(item_seq % g.n_items);
+            const int zb = (int)(item_seq % g.n_z);
+            if (!ptx::mbar_wait(&ifull[islot], (item_seq / g.n_items) & 1u, abort, kTimeoutNs)) break;
+            const int count = items[islot].count;
+            if (count < 0) break;
+            if (!ptx::mbar_wait(&zready[zb], (item_seq / g.n_z) & 1u, abort, kTimeoutNs)) break;
+            const float* zs = zbase + zb * zstride;
+            for (int j = tw; j < min(count, kTok); j += kTopkWarps)
+                topk_token(zs + j * P, P, top_k, lane, toks[islot * kTok + j], prim_out, weight_out);
+            __syncwarp();
+            if (lane == 0) {
+                ptx::mbar_arrive(&zfree[zb]);
+                ptx::mbar_arrive(&iempty[islot]);
             }
         }
-        __syncthreads();  // logits and queries are rewritten by the next item
+        return;
     }
-    if (tid == 0 && *abort) {
-        // Let every copy still in flight land before the CTA exits.
-        for (int64_t s = gs; s < total_stages && s < gs + kStages; ++s)
-            ptx::mbar_wait_drain(&full[s % kStages], (uint32_t)((s / kStages) & 1), kTimeoutNs);
-        atomicOr(status, STATUS_WAIT_TIMEOUT);
+
+    // ------------------------------------------------------------ compute warps
+    const int r_in_stage = tid / g.tpr;
+    const int seg = tid % g.tpr;
+    int64_t stage_seq = 0;
+    for (uint32_t item_seq = 0;; ++item_seq) {
+        const int islot = (int)(item_seq % g.n_items);
+        const int zb = (int)(item_seq % g.n_z);
+        ptx::mbar_wait(&ifull[islot], (item_seq / g.n_items) & 1u, abort, kTimeoutNs);
+        if (compute_sync_or(*abort != 0)) break;
+        const WorkItem w = items[islot];
+        if (w.count < 0) break;
+        const int nb = min(w.count, kTok);
+
+        // Queries of the item's tokens -> fp32, layout [token][half][chunk][4].
+        const T* qr = reinterpret_cast<const T*>(qraw + islot * g.qraw_bytes);
+        for (int i = tid; i < nb * dk; i += kCompute) {
+            const int j = i / dk, e = i - j * dk;
+            const int ch = e / EPC, h = (e % EPC) / 4;
+            qf[((j * H + h) * g.row_chunks + ch) * 4 + (e & 3)] = to_f32(qr[j * dk + e]);
+        }
+        // The logit buffer must have been released by the top-k warps.
+        ptx::mbar_wait(&zfree[zb], ((item_seq / g.n_z) & 1u) ^ 1u, abort, kTimeoutNs);
+        compute_sync_or(false);
+
+        float* zs = zbase + zb * zstride;
+        for (int st = 0; st < g.stages_per_item; ++st, ++stage_seq) {
+            const int slot = (int)(stage_seq % g.n_stages);
+            if (ptx::mbar_wait(&full[slot], (uint32_t)((stage_seq / g.n_stages) & 1), abort, kTimeoutNs)) {
+                const uint8_t* krow = ring + slot * kStageBytes + r_in_stage * g.row_bytes;
+                const int64_t row = (int64_t)st * g.rows_per_stage + r_in_stage;
+                switch (nb) {
+                    case 1: score_stage<T, 1>(krow, qf, g, seg, lane, row, P, scale, zs); break;
+                    case 2: score_stage<T, 2>(krow, qf, g, seg, lane, row, P, scale, zs); break;
+                    case 3: score_stage<T, 3>(krow, qf, g, seg, lane, row, P, scale, zs); break;
+                    case 4: score_stage<T, 4>(krow, qf, g, seg, lane, row, P, scale, zs); break;
+                    case 5: score_stage<T, 5>(krow, qf, g, seg, lane, row, P, scale, zs); break;
+                    case 6: score_stage<T, 6>(krow, qf, g, seg, lane, row, P, scale, zs); break;
+                    case 7: score_stage<T, 7>(krow, qf, g, seg, lane, row, P, scale, zs); break;
+                    default: score_stage<T, 8>(krow, qf, g, seg, lane, row, P, scale, zs); break;
+                }
+            }
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&empty[slot]);
+        }
+        // All logits written (and qf free for the next item) before the top-k warps read them.
+        if (compute_sync_or(*abort != 0)) break;
+        if (lane == 0) ptx::mbar_arrive(&zready[zb]);
     }
+}
+
+bool score_shape_supported(int dtype, int64_t P, int dk) {
+    const k3::Geometry g = k3::geometry(dtype, P, dk);
+    return g.tpr <= 32 && g.n_stages >= 2 && g.smem <= k3::kSmemLimit &&
+           g.rows_per_stage * g.row_bytes <= k3::kStageBytes;
 }
 
 cudaError_t launch_score(const LaunchCtx& c, const ScoreArgs& a) {
     const k3::Geometry g = k3::geometry(a.dtype, a.P, a.dk);
-    // Two CTAs per SM when their shared memory allows it.
-    const int per_sm = (2 * (g.smem + 1024) <= 228 * 1024) ? 2 : 1;
-    const int grid = c.num_sms * per_sm;
+    if (g.n_stages < 2 || g.smem > k3::kSmemLimit) return cudaErrorInvalidConfiguration;
     if (a.dtype == LOOKME_BF16) {
-        k3_score<__nv_bfloat16><<<grid, k3::kThreads, g.smem, c.stream>>>(
-            (const __nv_bfloat16*)a.q, (const __nv_bfloat16*)a.keys, a.P, a.dk, a.top_k, a.scale, a.work, a.n_work,
-            a.perm, a.use_slots, a.prim_out, a.weight_out, a.status, g);
+        k3_score<__nv_bfloat16><<<c.num_sms, k3::kThreads, g.smem, c.stream>>>(
+            (const __nv_bfloat16*)a.q, (const __nv_bfloat16*)a.keys, a.P, a.dk, a.top_k, a.scale, a.work,
+            a.counters, a.perm, a.use_slots, a.prim_out, a.weight_out, a.status, g);
     } else {
-        k3_score<float><<<grid, k3::kThreads, g.smem, c.stream>>>(
-            (const float*)a.q, (const float*)a.keys, a.P, a.dk, a.top_k, a.scale, a.work, a.n_work, a.perm,
+        k3_score<float><<<c.num_sms, k3::kThreads, g.smem, c.stream>>>(
+            (const float*)a.q, (const float*)a.keys, a.P, a.dk, a.top_k, a.scale, a.work, a.counters, a.perm,
             a.use_slots, a.prim_out, a.weight_out, a.status, g);
     }
     return cudaGetLastError();
@@ -254,9 +414,9 @@ cudaError_t launch_score(const LaunchCtx& c, const ScoreArgs& a) {
 
 cudaError_t configure_score_kernels() {
     cudaError_t e = cudaFuncSetAttribute(k3_score<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         227 * 1024);
+                                         k3::kSmemLimit);
     if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(k3_score<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+    return cudaFuncSetAttribute(k3_score<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, k3::kSmemLimit);
 }
 
 }  // namespace lookme

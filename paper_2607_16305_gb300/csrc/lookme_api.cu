@@ -303,6 +303,9 @@ lookme_status lookme_table_create(const lookme_table_desc* desc, lookme_table** 
     if (d.d_key % vec || d.d_value % vec)
         return fail(LOOKME_ERR_INVALID_ARG, "d_key and d_value must be multiples of %d for this dtype", vec);
     if (d.max_tokens < 0 || d.stage_slots < 0) return fail(LOOKME_ERR_INVALID_ARG, "negative size");
+    if (!score_shape_supported(d.dtype, d.n_prims, (int)d.d_key))
+        return fail(LOOKME_ERR_UNSUPPORTED, "n_prims %lld with d_key %lld does not fit the level-2 kernel's shared memory",
+                    (long long)d.n_prims, (long long)d.d_key);
     if ((int64_t)d.n_scenes * d.n_prims > ((int64_t)1 << 31) - 1)
         return fail(LOOKME_ERR_INVALID_ARG, "n_scenes * n_prims must fit in int32");
 
@@ -515,7 +518,7 @@ lookme_status lookme_lookup(lookme_table* t, const void* queries, int64_t N, int
     a.top_k = top_k;
     a.scale = (float)(1.0 / std::sqrt((double)dk));
     a.work = t->work;
-    a.n_work = t->counters;
+    a.counters = t->counters;
     a.perm = t->perm;
     a.use_slots = staged ? 1 : 0;
     a.prim_out = prim_out;

@@ -62,7 +62,7 @@ def _create(lib, **kw):
 @pytest.mark.parametrize("bad", [
     dict(n_scenes=0), dict(n_prims=0), dict(d_key=0), dict(d_value=0), dict(dtype=7), dict(residency=3),
     dict(reserved0=1), dict(d_key=12), dict(d_value=20, dtype=0), dict(d_key=6, dtype=1), dict(n_scenes=10**6),
-    dict(n_prims=4096), dict(max_tokens=-1), dict(device=-1),
+    dict(n_prims=4096), dict(max_tokens=-1), dict(device=-1), dict(d_key=2048),
 ])
 def test_create_rejects_bad_desc(lib, bad):
     from paper_2607_16305_gb300 import lookme
