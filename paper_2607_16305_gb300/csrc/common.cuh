@@ -135,6 +135,10 @@ struct ScoreArgs {
 cudaError_t launch_score(const LaunchCtx& c, const ScoreArgs& a);
 // Whether the level-2 kernel's shared-memory plan fits this table shape.
 bool score_shape_supported(int dtype, int64_t P, int dk);
+// Level 2 on tcgen05 (bf16 tables): tmap_keys is the CUtensorMap of the key
+// rows ([rows][d_k], box 64 x 128, 128-byte swizzle).
+cudaError_t launch_score_tc(const LaunchCtx& c, const void* tmap_keys, const ScoreArgs& a);
+bool score_tc_shape_supported(int64_t P, int dk);
 // K5
 cudaError_t launch_select(const LaunchCtx& c, const float* priority, int64_t N, const int64_t* seg_off_host,
                           int n_seg, double keep_ratio, uint8_t* mask, int32_t* sel);
@@ -165,6 +169,7 @@ cudaError_t launch_stage(const LaunchCtx& c, const void* keys_host_mapped, void*
 cudaError_t configure_route_kernels();
 cudaError_t configure_bucket_kernel();
 cudaError_t configure_score_kernels();
+cudaError_t configure_score_tc_kernel();
 // load-time
 cudaError_t launch_centroid_mean(const LaunchCtx& c, int dtype, const void* keys, int64_t n, int64_t P, int dk,
                                  void* cent);

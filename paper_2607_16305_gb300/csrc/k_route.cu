@@ -193,6 +193,8 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
     const int nt1 = min(n_tiles, nt0 + tiles_per_cta);
 
     if (threadIdx.x == 0) {
+        ptx::prefetch_tmap(&tmap_q);
+        ptx::prefetch_tmap(&tmap_c);
         for (int i = 0; i < STAGES; ++i) {
             ptx::mbar_init(&full[i], 1);
             ptx::mbar_init(&empty[i], 1);

@@ -28,6 +28,7 @@
 // reduction makes the abort decision uniform; every wait is bounded.
 #include "common.cuh"
 #include "sm100.cuh"
+#include "topk.cuh"
 
 namespace lookme {
 
@@ -140,71 +141,6 @@ __device__ __forceinline__ void score_stage(const uint8_t* krow, const float* qf
     }
 }
 
-// Inverse of orderable(): the float whose order key is u.
-__device__ __forceinline__ float from_orderable(uint32_t u) {
-    return __uint_as_float((u & 0x80000000u) ? (u & 0x7FFFFFFFu) : ~u);
-}
-
-// Top-k of z[0..P) by one warp (larger z first, lower index on ties) and the
-// softmax over the selected logits; writes prim/weight of token t.
-__device__ __forceinline__ void topk_token(const float* z, int64_t P, int top_k, int lane, int64_t t,
-                                           int32_t* prim_out, float* weight_out) {
-    // Each lane keeps the best untaken element of its slice p = lane + 32 i.
-    uint64_t taken = 0ull;
-    auto local_best = [&](uint32_t& key, uint32_t& pb) {
-        key = 0u;
-        pb = 0xFFFFFFFFu;
-        int i = 0;
-        for (int64_t p = lane; p < P; p += 32, ++i) {
-            if (!((taken >> i) & 1ull)) {
-                const uint32_t k = orderable(z[p]);
-                if (pb == 0xFFFFFFFFu || k > key) {
-                    key = k;
-                    pb = (uint32_t)p;
-                }
-            }
-        }
-    };
-    uint32_t key, pb;
-    local_best(key, pb);
-    float my_z[2] = {0.f, 0.f};  // output slots lane and lane + 32
-    int my_p[2] = {0, 0};
-    for (int kk = 0; kk < top_k; ++kk) {
-        const uint32_t kmax = __reduce_max_sync(0xFFFFFFFFu, pb == 0xFFFFFFFFu ? 0u : key);
-        const uint32_t pmin = __reduce_min_sync(0xFFFFFFFFu, (pb != 0xFFFFFFFFu && key == kmax) ? pb : 0xFFFFFFFFu);
-        if ((kk & 31) == lane) {
-            if (kk < 32) {
-                my_z[0] = from_orderable(kmax);
-                my_p[0] = (int)pmin;
-            } else {
-                my_z[1] = from_orderable(kmax);
-                my_p[1] = (int)pmin;
-            }
-        }
-        if (pmin != 0xFFFFFFFFu && (int)(pmin & 31u) == lane) {
-            taken |= 1ull << (pmin >> 5);
-            local_best(key, pb);
-        }
-    }
-    const float zmax = __shfl_sync(0xFFFFFFFFu, my_z[0], 0);
-    float e[2];
-    float sum = 0.f;
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-        e[h] = (h * 32 + lane < top_k) ? expf(my_z[h] - zmax) : 0.f;
-        sum += e[h];
-    }
-#pragma unroll
-    for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-        const int j = h * 32 + lane;
-        if (j < top_k) {
-            prim_out[t * top_k + j] = my_p[h];
-            weight_out[t * top_k + j] = e[h] / sum;
-        }
-    }
-}
 }  // namespace k3
 
 template <typename T>
@@ -331,7 +267,7 @@ __global__ void __launch_bounds__(k3::kThreads, 1)
             if (!ptx::mbar_wait(&zready[zb], (item_seq / g.n_z) & 1u, abort, kTimeoutNs)) break;
             const float* zs = zbase + zb * zstride;
             for (int j = tw; j < min(count, kTok); j += kTopkWarps)
-                topk_token(zs + j * P, P, top_k, lane, toks[islot * kTok + j], prim_out, weight_out);
+                topk_any(zs + j * P, P, top_k, lane, toks[islot * kTok + j], prim_out, weight_out);
             __syncwarp();
             if (lane == 0) {
                 ptx::mbar_arrive(&zfree[zb]);

@@ -99,6 +99,8 @@ struct lookme_table {
     size_t esz = 2;
     int num_sms = 0;
     bool tc_route = false;  // level 1 on tcgen05
+    bool tc_score = false;  // level 2 on tcgen05
+    CUtensorMap tmap_keys;  // key rows (table or slot cache) for the tcgen05 level-2 kernel
 
     // storage
     void* keys = nullptr;       // device, or device-mapped pinned host
@@ -322,16 +324,21 @@ lookme_status lookme_table_create(const lookme_table_desc* desc, lookme_table** 
     t->esz = d.dtype == LOOKME_BF16 ? 2 : 4;
     cudaDeviceGetAttribute(&t->num_sms, cudaDevAttrMultiProcessorCount, d.device);
     t->tc_route = d.dtype == LOOKME_BF16 && d.d_key <= kRouteTcMaxDk;
-    // Validation switch: LOOKME_ROUTE=simt routes bf16 tables on the CUDA-core
-    // kernel too, so the two level-1 kernels can be checked against each other.
+    t->tc_score = d.dtype == LOOKME_BF16 && score_tc_shape_supported(d.n_prims, (int)d.d_key);
+    // Validation switches: LOOKME_ROUTE=simt / LOOKME_SCORE=simt run bf16 tables
+    // on the CUDA-core level-1 / level-2 kernels too, so each pair of kernels
+    // can be checked against each other.
     if (const char* env = getenv("LOOKME_ROUTE")) {
         if (strcmp(env, "simt") == 0) t->tc_route = false;
+    }
+    if (const char* env = getenv("LOOKME_SCORE")) {
+        if (strcmp(env, "simt") == 0) t->tc_score = false;
     }
     t->loaded.assign(d.n_scenes, 0);
 
     cudaError_t e;
     if ((e = configure_route_kernels()) != cudaSuccess || (e = configure_bucket_kernel()) != cudaSuccess ||
-        (e = configure_score_kernels()) != cudaSuccess) {
+        (e = configure_score_kernels()) != cudaSuccess || (e = configure_score_tc_kernel()) != cudaSuccess) {
         destroy_table(t);
         return fail(LOOKME_ERR_CUDA, "kernel configuration: %s", cudaGetErrorString(e));
     }
@@ -363,6 +370,14 @@ lookme_status lookme_table_create(const lookme_table_desc* desc, lookme_table** 
         cudaMemset(t->status, 0, 256) != cudaSuccess) {
         destroy_table(t);
         return fail(LOOKME_ERR_CUDA, "table initialisation failed");
+    }
+    if (t->tc_score) {
+        const bool staged = d.residency == LOOKME_RES_HOST_STAGED;
+        const int64_t rows = (staged ? t->n_slots : d.n_scenes) * d.n_prims;
+        if (!encode_bf16_2d(&t->tmap_keys, staged ? t->slots : t->keys, rows, d.d_key, 128)) {
+            destroy_table(t);
+            return fail(LOOKME_ERR_CUDA, "cuTensorMapEncodeTiled failed for the keys");
+        }
     }
     if (t->tc_route) {
         for (int i = 0; i < 3; ++i) {
@@ -524,7 +539,7 @@ lookme_status lookme_lookup(lookme_table* t, const void* queries, int64_t N, int
     a.prim_out = prim_out;
     a.weight_out = weight_out;
     a.status = t->status;
-    st = launch(t, s, KID_SCORE, [&] { return launch_score(ctx, a); });
+    st = launch(t, s, KID_SCORE, [&] { return t->tc_score ? launch_score_tc(ctx, &t->tmap_keys, a) : launch_score(ctx, a); });
     if (st != LOOKME_OK) return st;
     t->last_tokens = N;
     return LOOKME_OK;

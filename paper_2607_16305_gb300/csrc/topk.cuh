@@ -1,0 +1,149 @@
+// Warp-level top-k + softmax of one token's level-2 logits (Sec. "Level-2:
+// scene-primitive retrieval": I = top-k of the logits, weights = softmax over
+// the selected), shared by the level-2 kernels.
+#pragma once
+
+#include "common.cuh"
+
+namespace lookme {
+namespace k3 {
+
+// Inverse of orderable(): the float whose order key is u.
+__device__ __forceinline__ float from_orderable(uint32_t u) {
+    return __uint_as_float((u & 0x80000000u) ? (u & 0x7FFFFFFFu) : ~u);
+}
+
+// Top-k of z[0..P) by one warp (larger z first, lower index on ties) and the
+// softmax over the selected logits; writes prim/weight of token t.
+__device__ __forceinline__ void topk_token(const float* z, int64_t P, int top_k, int lane, int64_t t,
+                                           int32_t* prim_out, float* weight_out) {
+    // Each lane keeps the best untaken element of its slice p = lane + 32 i.
+    uint64_t taken = 0ull;
+    auto local_best = [&](uint32_t& key, uint32_t& pb) {
+        key = 0u;
+        pb = 0xFFFFFFFFu;
+        int i = 0;
+        for (int64_t p = lane; p < P; p += 32, ++i) {
+            if (!((taken >> i) & 1ull)) {
+                const uint32_t k = orderable(z[p]);
+                if (pb == 0xFFFFFFFFu || k > key) {
+                    key = k;
+                    pb = (uint32_t)p;
+                }
+            }
+        }
+    };
+    uint32_t key, pb;
+    local_best(key, pb);
+    float my_z[2] = {0.f, 0.f};  // output slots lane and lane + 32
+    int my_p[2] = {0, 0};
+    for (int kk = 0; kk < top_k; ++kk) {
+        const uint32_t kmax = __reduce_max_sync(0xFFFFFFFFu, pb == 0xFFFFFFFFu ? 0u : key);
+        const uint32_t pmin = __reduce_min_sync(0xFFFFFFFFu, (pb != 0xFFFFFFFFu && key == kmax) ? pb : 0xFFFFFFFFu);
+        if ((kk & 31) == lane) {
+            if (kk < 32) {
+                my_z[0] = from_orderable(kmax);
+                my_p[0] = (int)pmin;
+            } else {
+                my_z[1] = from_orderable(kmax);
+                my_p[1] = (int)pmin;
+            }
+        }
+        if (pmin != 0xFFFFFFFFu && (int)(pmin & 31u) == lane) {
+            taken |= 1ull << (pmin >> 5);
+            local_best(key, pb);
+        }
+    }
+    const float zmax = __shfl_sync(0xFFFFFFFFu, my_z[0], 0);
+    float e[2];
+    float sum = 0.f;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        e[h] = (h * 32 + lane < top_k) ? expf(my_z[h] - zmax) : 0.f;
+        sum += e[h];
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int j = h * 32 + lane;
+        if (j < top_k) {
+            prim_out[t * top_k + j] = my_p[h];
+            weight_out[t * top_k + j] = e[h] / sum;
+        }
+    }
+}
+// Register-resident variant for N_p <= 32 * PPL: each lane holds the order
+// keys of its elements p = 32 i + lane, so a round is an unrolled scan of
+// PPL registers plus two warp reductions.  Same result as topk_token.
+template <int PPL>
+__device__ __forceinline__ void topk_token_regs(const float* z, int64_t P, int top_k, int lane, int64_t t,
+                                                int32_t* prim_out, float* weight_out) {
+    uint32_t key[PPL];
+#pragma unroll
+    for (int i = 0; i < PPL; ++i) {
+        const int64_t p = (int64_t)i * 32 + lane;
+        key[i] = p < P ? max(orderable(z[p]), 1u) : 0u;  // 0 marks "no element"
+    }
+    uint32_t taken = 0u;
+    float my_z[2] = {0.f, 0.f};
+    int my_p[2] = {0, 0};
+    for (int kk = 0; kk < top_k; ++kk) {
+        uint32_t bk = 0u;
+        int bi = -1;
+#pragma unroll
+        for (int i = 0; i < PPL; ++i) {
+            if (!((taken >> i) & 1u) && key[i] > bk) {  // strict: the lowest i (lowest p) wins ties
+                bk = key[i];
+                bi = i;
+            }
+        }
+        const uint32_t kmax = __reduce_max_sync(0xFFFFFFFFu, bk);
+        const uint32_t pmin = __reduce_min_sync(0xFFFFFFFFu, (bi >= 0 && bk == kmax) ? (uint32_t)(bi * 32 + lane)
+                                                                                     : 0xFFFFFFFFu);
+        if (pmin != 0xFFFFFFFFu && (int)(pmin & 31u) == lane) taken |= 1u << (pmin >> 5);
+        if ((kk & 31) == lane) {
+            const float zz = pmin != 0xFFFFFFFFu ? z[pmin] : 0.f;
+            if (kk < 32) {
+                my_z[0] = zz;
+                my_p[0] = (int)pmin;
+            } else {
+                my_z[1] = zz;
+                my_p[1] = (int)pmin;
+            }
+        }
+    }
+    const float zmax = __shfl_sync(0xFFFFFFFFu, my_z[0], 0);
+    float e[2];
+    float sum = 0.f;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        e[h] = (h * 32 + lane < top_k) ? expf(my_z[h] - zmax) : 0.f;
+        sum += e[h];
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int j = h * 32 + lane;
+        if (j < top_k) {
+            prim_out[t * top_k + j] = my_p[h];
+            weight_out[t * top_k + j] = e[h] / sum;
+        }
+    }
+}
+
+// Top-k of one token, picking the register-resident variant when N_p allows.
+__device__ __forceinline__ void topk_any(const float* z, int64_t P, int top_k, int lane, int64_t t,
+                                         int32_t* prim_out, float* weight_out) {
+    if (P <= 32) topk_token_regs<1>(z, P, top_k, lane, t, prim_out, weight_out);
+    else if (P <= 64) topk_token_regs<2>(z, P, top_k, lane, t, prim_out, weight_out);
+    else if (P <= 128) topk_token_regs<4>(z, P, top_k, lane, t, prim_out, weight_out);
+    else if (P <= 256) topk_token_regs<8>(z, P, top_k, lane, t, prim_out, weight_out);
+    else if (P <= 512) topk_token_regs<16>(z, P, top_k, lane, t, prim_out, weight_out);
+    else if (P <= 1024) topk_token_regs<32>(z, P, top_k, lane, t, prim_out, weight_out);
+    else topk_token(z, P, top_k, lane, t, prim_out, weight_out);
+}
+
+}  // namespace k3
+}  // namespace lookme

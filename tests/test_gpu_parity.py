@@ -232,3 +232,16 @@ def test_graph_capture_replay(oracle, lookme_lib):
         torch.cuda.synchronize()
         assert torch.equal(scene, s_ref) and torch.equal(prim, p_ref) and torch.equal(weight, w_ref)
         assert torch.equal(hg, h_ref)
+
+
+@pytest.mark.parametrize("case", ["single_image", "s6"])
+def test_cuda_core_variants(oracle, lookme_lib, monkeypatch, case):
+    """The CUDA-core level-1 and level-2 kernels (selected per table by the
+    LOOKME_ROUTE / LOOKME_SCORE switches) against the oracle on bf16 tables."""
+    monkeypatch.setenv("LOOKME_ROUTE", "simt")
+    monkeypatch.setenv("LOOKME_SCORE", "simt")
+    if case == "single_image":
+        w = W.WORKLOADS["single_image"]
+    else:
+        w = W.small("s6_simt", **dict(SMALL_CASES)["s6"])
+    run_case(oracle, lookme_lib, w)
