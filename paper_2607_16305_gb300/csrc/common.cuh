@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "lookme.h"
 
 namespace lookme {
@@ -91,6 +93,31 @@ __device__ __forceinline__ int32_t unpack_scene(unsigned long long key, int64_t 
 struct WorkItem {
     int32_t scene, begin, count, slot;
 };
+
+// ---------------------------------------------- programmatic dependent launch
+// Every per-call kernel is launched with programmatic stream serialisation:
+// it may start while its predecessor on the stream is still running, lets its
+// own successor start early (pdl_trigger), and waits for the predecessor's
+// completion and memory (pdl_wait) before it touches any data a predecessor
+// produces or consumes.  Both are no-ops for a normal launch.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                       Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // ------------------------------------------------------------ launch params
 struct LaunchCtx {

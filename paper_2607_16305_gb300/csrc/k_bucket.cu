@@ -67,6 +67,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     extern __shared__ int cnt[];  // [S]: counts, then running token offsets
     __shared__ int3 warp_buf[33];
     __shared__ int max_bucket;
+    pdl_trigger();
+    pdl_wait();
     const int tid = threadIdx.x;
     for (int s = tid; s < S; s += kThreads) cnt[s] = 0;
     if (tid == 0) max_bucket = 0;
@@ -129,8 +131,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 cudaError_t launch_bucket(const LaunchCtx& c, const unsigned long long* best, int64_t N, int64_t S,
                           int32_t* scene_out, int32_t* perm, WorkItem* work, int32_t* routed, int32_t* counters) {
     const size_t smem = (size_t)S * sizeof(int);
-    k2_bucket<<<1, kThreads, smem, c.stream>>>(best, N, (int)S, scene_out, perm, work, routed, counters);
-    return cudaGetLastError();
+    return launch_pdl(k2_bucket, dim3(1), dim3(kThreads), smem, c.stream, best, N, (int)S, scene_out, perm, work,
+                      routed, counters);
 }
 
 cudaError_t configure_bucket_kernel() {

@@ -64,6 +64,8 @@ __global__ void __launch_bounds__(k5::kThreads, 1) k5_select(const __grid_consta
     __shared__ int scan_buf[33];
     __shared__ uint32_t sh_prefix;
     __shared__ int sh_remaining;
+    pdl_trigger();
+    pdl_wait();
     const int seg = blockIdx.x;
     const int64_t b = p.off[seg], len = p.off[seg + 1] - p.off[seg];
     const int64_t r = (int64_t)floor((double)len * p.keep_ratio);
@@ -154,8 +156,7 @@ cudaError_t launch_select(const LaunchCtx& c, const float* priority, int64_t N, 
     p.keep_ratio = keep_ratio;
     p.n_seg = n_seg;
     for (int i = 0; i <= n_seg; ++i) p.off[i] = seg_off_host ? seg_off_host[i] : (i == 0 ? 0 : N);
-    k5_select<<<n_seg, k5::kThreads, 0, c.stream>>>(p);
-    return cudaGetLastError();
+    return launch_pdl(k5_select, dim3(n_seg), dim3(k5::kThreads), 0, c.stream, p);
 }
 
 // ---------------------------------------------------------------- K4 inject
@@ -184,6 +185,8 @@ __global__ void __launch_bounds__(k4::kThreads) k4_inject(const __grid_constant_
     constexpr int BATCH = 8;  // value rows in flight per thread
     __shared__ const uint4* rows[LOOKME_MAX_TOP_K];
     __shared__ float w[LOOKME_MAX_TOP_K];
+    pdl_trigger();
+    pdl_wait();
     const int64_t t = p.sel[blockIdx.x];
     const int64_t s = min(max((int64_t)p.scene[t], (int64_t)0), p.S - 1);
     for (int j = threadIdx.x; j < p.top_k; j += blockDim.x) {
@@ -246,10 +249,8 @@ cudaError_t launch_inject(const LaunchCtx& c, const InjectArgs& a) {
     int threads = (chunks + 31) / 32 * 32;
     if (threads > k4::kThreads) threads = k4::kThreads;
     if (a.dtype == LOOKME_BF16)
-        k4_inject<__nv_bfloat16><<<(unsigned)a.n_sel, threads, 0, c.stream>>>(p);
-    else
-        k4_inject<float><<<(unsigned)a.n_sel, threads, 0, c.stream>>>(p);
-    return cudaGetLastError();
+        return launch_pdl(k4_inject<__nv_bfloat16>, dim3((unsigned)a.n_sel), dim3(threads), 0, c.stream, p);
+    return launch_pdl(k4_inject<float>, dim3((unsigned)a.n_sel), dim3(threads), 0, c.stream, p);
 }
 
 }  // namespace lookme

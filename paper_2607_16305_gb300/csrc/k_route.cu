@@ -19,6 +19,8 @@ template <typename T>
 __global__ void __launch_bounds__(256) k0_prep(const T* __restrict__ q, int64_t N, int dk,
                                                float* __restrict__ qnorm, float* __restrict__ qnorm_out,
                                                unsigned long long* __restrict__ best) {
+    pdl_trigger();
+    pdl_wait();
     const int64_t t = (int64_t)blockIdx.x * 8 + threadIdx.x / 32;
     const int lane = threadIdx.x % 32;
     if (t >= N) return;
@@ -47,10 +49,9 @@ cudaError_t launch_prep(const LaunchCtx& c, int dtype, const void* q, int64_t N,
     if (N == 0) return cudaSuccess;
     dim3 grid((unsigned)((N + 7) / 8));
     if (dtype == LOOKME_BF16)
-        k0_prep<__nv_bfloat16><<<grid, 256, 0, c.stream>>>((const __nv_bfloat16*)q, N, dk, qnorm, qnorm_out, best);
-    else
-        k0_prep<float><<<grid, 256, 0, c.stream>>>((const float*)q, N, dk, qnorm, qnorm_out, best);
-    return cudaGetLastError();
+        return launch_pdl(k0_prep<__nv_bfloat16>, grid, dim3(256), 0, c.stream, (const __nv_bfloat16*)q, N, dk, qnorm,
+                          qnorm_out, best);
+    return launch_pdl(k0_prep<float>, grid, dim3(256), 0, c.stream, (const float*)q, N, dk, qnorm, qnorm_out, best);
 }
 
 // Score of token row against scene s from the raw dot product.
@@ -72,6 +73,8 @@ __global__ void __launch_bounds__(256) k1_route_simt(const T* __restrict__ q, co
                                                      unsigned long long* __restrict__ best) {
     __shared__ float As[16][64 + 4];
     __shared__ float Bs[16][64 + 4];
+    pdl_trigger();
+    pdl_wait();
     const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
     const int64_t row0 = (int64_t)blockIdx.y * 64, col0 = (int64_t)blockIdx.x * 64;
     float acc[4][4];
@@ -136,12 +139,10 @@ cudaError_t launch_route_simt(const LaunchCtx& c, int dtype, const void* q, cons
     if (N == 0) return cudaSuccess;
     dim3 grid((unsigned)((S + 63) / 64), (unsigned)((N + 63) / 64));
     if (dtype == LOOKME_BF16)
-        k1_route_simt<__nv_bfloat16><<<grid, 256, 0, c.stream>>>(
-            (const __nv_bfloat16*)q, (const __nv_bfloat16*)cent, N, S, dk, inv_cnorm, bias, qnorm, best);
-    else
-        k1_route_simt<float><<<grid, 256, 0, c.stream>>>((const float*)q, (const float*)cent, N, S, dk,
-                                                         inv_cnorm, bias, qnorm, best);
-    return cudaGetLastError();
+        return launch_pdl(k1_route_simt<__nv_bfloat16>, grid, dim3(256), 0, c.stream, (const __nv_bfloat16*)q,
+                          (const __nv_bfloat16*)cent, N, S, dk, inv_cnorm, bias, qnorm, best);
+    return launch_pdl(k1_route_simt<float>, grid, dim3(256), 0, c.stream, (const float*)q, (const float*)cent, N, S,
+                      dk, inv_cnorm, bias, qnorm, best);
 }
 
 // ---------------------------------------------------- K1 on tcgen05 (bf16)
@@ -208,6 +209,10 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
         *abort = 0;
         ptx::fence_mbar_init();
     }
+    pdl_trigger();
+    // TMEM is allocated only after the predecessor has completed, so a CTA
+    // that holds TMEM never waits on an earlier kernel.
+    pdl_wait();
     if (warp == 1) ptx::tmem_alloc(tmem_slot, 2 * BN);
     ptx::tc_fence_before();
     __syncthreads();
@@ -366,9 +371,8 @@ static cudaError_t launch_route_tc_t(const LaunchCtx& c, const void* tmap_q, con
     CUtensorMap mq, mc;
     memcpy(&mq, tmap_q, sizeof(CUtensorMap));
     memcpy(&mc, tmap_c, sizeof(CUtensorMap));
-    k1_route_tc<BN, STAGES><<<dim3(m_tiles, splits), kThreads, smem, c.stream>>>(
-        mq, mc, N, S, dk, per, inv_cnorm, bias, qnorm, best, status);
-    return cudaGetLastError();
+    return launch_pdl(k1_route_tc<BN, STAGES>, dim3(m_tiles, splits), dim3(kThreads), (size_t)smem, c.stream, mq, mc,
+                      N, S, dk, per, inv_cnorm, bias, qnorm, best, status);
 }
 
 cudaError_t launch_route_tc(const LaunchCtx& c, const void* tmap_q, const void* const tmap_c[3], int64_t N,

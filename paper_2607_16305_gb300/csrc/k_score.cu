@@ -168,6 +168,8 @@ __global__ void __launch_bounds__(k3::kThreads, 1)
     volatile int* abort = reinterpret_cast<volatile int*>(toks + kMaxItemSlots * kTok);
 
     const int tid = threadIdx.x, lane = tid % 32, warp = tid / 32;
+    pdl_trigger();
+    pdl_wait();
     const int n_work = counters[0];
     const int64_t zstride = (int64_t)kTok * P;
 
@@ -336,16 +338,13 @@ bool score_shape_supported(int dtype, int64_t P, int dk) {
 cudaError_t launch_score(const LaunchCtx& c, const ScoreArgs& a) {
     const k3::Geometry g = k3::geometry(a.dtype, a.P, a.dk);
     if (g.n_stages < 2 || g.smem > k3::kSmemLimit) return cudaErrorInvalidConfiguration;
-    if (a.dtype == LOOKME_BF16) {
-        k3_score<__nv_bfloat16><<<c.num_sms, k3::kThreads, g.smem, c.stream>>>(
-            (const __nv_bfloat16*)a.q, (const __nv_bfloat16*)a.keys, a.P, a.dk, a.top_k, a.scale, a.work,
-            a.counters, a.perm, a.use_slots, a.prim_out, a.weight_out, a.status, g);
-    } else {
-        k3_score<float><<<c.num_sms, k3::kThreads, g.smem, c.stream>>>(
-            (const float*)a.q, (const float*)a.keys, a.P, a.dk, a.top_k, a.scale, a.work, a.counters, a.perm,
-            a.use_slots, a.prim_out, a.weight_out, a.status, g);
-    }
-    return cudaGetLastError();
+    if (a.dtype == LOOKME_BF16)
+        return launch_pdl(k3_score<__nv_bfloat16>, dim3(c.num_sms), dim3(k3::kThreads), (size_t)g.smem, c.stream,
+                          (const __nv_bfloat16*)a.q, (const __nv_bfloat16*)a.keys, a.P, a.dk, a.top_k, a.scale, a.work,
+                          a.counters, a.perm, a.use_slots, a.prim_out, a.weight_out, a.status, g);
+    return launch_pdl(k3_score<float>, dim3(c.num_sms), dim3(k3::kThreads), (size_t)g.smem, c.stream,
+                      (const float*)a.q, (const float*)a.keys, a.P, a.dk, a.top_k, a.scale, a.work, a.counters, a.perm,
+                      a.use_slots, a.prim_out, a.weight_out, a.status, g);
 }
 
 cudaError_t configure_score_kernels() {

@@ -121,13 +121,17 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
     volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int tid = threadIdx.x, lane = tid % 32, warp = tid / 32;
+    if (tid == 0) ptx::prefetch_tmap(&tmap_keys);
+    pdl_trigger();
+    // The work list is the predecessor's output; TMEM is allocated only after
+    // this wait, so a CTA that holds TMEM never waits on an earlier kernel.
+    pdl_wait();
     const int n_work = counters[0];
     const int G = gridDim.x;
     const int my_items = n_work > (int)blockIdx.x ? (n_work - (int)blockIdx.x + G - 1) / G : 0;
     if (my_items == 0) return;  // uniform for the CTA: nothing allocated yet
 
     if (tid == 0) {
-        ptx::prefetch_tmap(&tmap_keys);
         for (int i = 0; i < g.n_stages; ++i) {
             ptx::mbar_init(&full[i], 1);
             ptx::mbar_init(&empty[i], 1);
@@ -359,10 +363,9 @@ cudaError_t launch_score_tc(const LaunchCtx& c, const void* tmap_keys, const Sco
     if (!score_tc_shape_supported(a.P, a.dk)) return cudaErrorInvalidConfiguration;
     CUtensorMap mk;
     memcpy(&mk, tmap_keys, sizeof(CUtensorMap));
-    k3_score_tc<<<c.num_sms, k3tc::kThreads, g.smem, c.stream>>>(
-        mk, (const __nv_bfloat16*)a.q, a.P, a.dk, a.top_k, a.scale, a.work, a.counters, a.perm, a.use_slots,
-        a.prim_out, a.weight_out, a.status, g);
-    return cudaGetLastError();
+    return launch_pdl(k3_score_tc, dim3(c.num_sms), dim3(k3tc::kThreads), (size_t)g.smem, c.stream, mk,
+                      (const __nv_bfloat16*)a.q, a.P, a.dk, a.top_k, a.scale, a.work, (const int32_t*)a.counters, a.perm,
+                      a.use_slots, a.prim_out, a.weight_out, a.status, g);
 }
 
 cudaError_t configure_score_tc_kernel() {

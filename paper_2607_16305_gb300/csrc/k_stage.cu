@@ -14,6 +14,8 @@ __global__ void __launch_bounds__(256) k6_stage(const uint4* __restrict__ keys_h
                                                 int64_t block_vecs, int64_t n_slots,
                                                 const int32_t* __restrict__ routed,
                                                 const int32_t* __restrict__ counters) {
+    pdl_trigger();
+    pdl_wait();
     const int64_t n_routed = min((int64_t)counters[1], n_slots);
     const int64_t total = n_routed * block_vecs;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -38,9 +40,8 @@ __global__ void __launch_bounds__(256) k6_stage(const uint4* __restrict__ keys_h
 
 cudaError_t launch_stage(const LaunchCtx& c, const void* keys_host_mapped, void* slots, int64_t block_bytes,
                          int64_t n_slots, const int32_t* routed, const int32_t* counters) {
-    k6_stage<<<c.num_sms * 8, 256, 0, c.stream>>>((const uint4*)keys_host_mapped, (uint4*)slots, block_bytes / 16,
-                                                   n_slots, routed, counters);
-    return cudaGetLastError();
+    return launch_pdl(k6_stage, dim3(c.num_sms * 8), dim3(256), 0, c.stream, (const uint4*)keys_host_mapped,
+                      (uint4*)slots, block_bytes / 16, n_slots, routed, counters);
 }
 
 }  // namespace lookme
