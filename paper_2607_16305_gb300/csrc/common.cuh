@@ -25,6 +25,7 @@ enum KernelId : int32_t {
     KID_CENTROID = 8,    // load-time: centroid = mean of keys
     KID_CNORM = 9,       // load-time: 1 / ||centroid||
     KID_ROUTE_DECODE = 10,  // argmax key -> scene id (allocation-free routing)
+    KID_SELECT_INJECT = 11, // K5 + K4 fused for short segments
     KID_COUNT
 };
 
@@ -187,6 +188,11 @@ struct InjectArgs {
     void* hidden[LOOKME_MAX_LAYERS];
 };
 cudaError_t launch_inject(const LaunchCtx& c, const InjectArgs& a);
+// K5 + K4 in one kernel (one CTA per token) for segments of at most
+// kFusedMaxSegment tokens when the kept-id list is not requested.
+constexpr int64_t kFusedMaxSegment = 8192;
+cudaError_t launch_select_inject(const LaunchCtx& c, const InjectArgs& a, const float* priority,
+                                 const int64_t* seg_off_host, int n_seg, double keep_ratio, uint8_t* mask);
 // K6
 cudaError_t launch_stage(const LaunchCtx& c, const void* keys_host_mapped, void* slots, int64_t block_bytes,
                          int64_t n_slots, const int32_t* routed, const int32_t* counters);

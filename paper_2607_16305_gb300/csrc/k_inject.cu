@@ -179,15 +179,13 @@ struct Params {
 };
 }  // namespace k4
 
+// Gather + weighted sum + residual add for token t by one CTA.
 template <typename T>
-__global__ void __launch_bounds__(k4::kThreads) k4_inject(const __grid_constant__ k4::Params p) {
+__device__ __forceinline__ void inject_token(const k4::Params& p, int64_t t) {
     constexpr int EPC = Vec16<T>::N;
     constexpr int BATCH = 8;  // value rows in flight per thread
     __shared__ const uint4* rows[LOOKME_MAX_TOP_K];
     __shared__ float w[LOOKME_MAX_TOP_K];
-    pdl_trigger();
-    pdl_wait();
-    const int64_t t = p.sel[blockIdx.x];
     const int64_t s = min(max((int64_t)p.scene[t], (int64_t)0), p.S - 1);
     for (int j = threadIdx.x; j < p.top_k; j += blockDim.x) {
         const int64_t pr = min(max((int64_t)p.prim[t * p.top_k + j], (int64_t)0), p.P - 1);
@@ -227,6 +225,86 @@ __global__ void __launch_bounds__(k4::kThreads) k4_inject(const __grid_constant_
             *h = Vec16<T>::pack(f);
         }
     }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(k4::kThreads) k4_inject(const __grid_constant__ k4::Params p) {
+    pdl_trigger();
+    pdl_wait();
+    inject_token<T>(p, p.sel[blockIdx.x]);
+}
+
+// Selection fused into the injection (segments of at most kFusedMaxSegment
+// tokens): one CTA per token computes the token's rank in its segment,
+//   rank_t = #{ j : pi_j > pi_t, or pi_j == pi_t and j < t },
+// which orders tokens exactly like the radix selection (larger priority
+// first, lower index on ties); the token is kept iff rank_t < r.  Kept tokens
+// are injected by the same CTA.
+template <typename T>
+__global__ void __launch_bounds__(k4::kThreads) k45_select_inject(const __grid_constant__ k4::Params p,
+                                                                  const __grid_constant__ k5::Params sp) {
+    __shared__ int warp_cnt[k4::kThreads / 32];
+    pdl_trigger();
+    pdl_wait();
+    const int64_t t = blockIdx.x;
+    int lo = 0, hi = sp.n_seg;  // segment: off[lo] <= t < off[lo + 1]
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) / 2;
+        if (sp.off[mid] <= t) lo = mid;
+        else hi = mid;
+    }
+    const int64_t b = sp.off[lo], len = sp.off[lo + 1] - b;
+    const int64_t r = (int64_t)floor((double)len * sp.keep_ratio);
+    bool keep = r >= len;
+    if (r > 0 && r < len) {
+        const uint32_t kt = k5::prio_key(sp.priority[t]);
+        int cnt = 0;
+        for (int64_t j = threadIdx.x; j < len; j += blockDim.x) {
+            const uint32_t kj = k5::prio_key(sp.priority[b + j]);
+            cnt += (kj > kt) || (kj == kt && b + j < t);
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) cnt += __shfl_xor_sync(0xFFFFFFFFu, cnt, o);
+        if ((threadIdx.x & 31) == 0) warp_cnt[threadIdx.x / 32] = cnt;
+        __syncthreads();
+        int total = 0;
+        for (int i = 0; i < (int)(blockDim.x / 32); ++i) total += warp_cnt[i];
+        keep = total < r;
+    }
+    if (threadIdx.x == 0 && sp.mask) sp.mask[t] = (uint8_t)keep;
+    if (keep) inject_token<T>(p, t);
+}
+
+cudaError_t launch_select_inject(const LaunchCtx& c, const InjectArgs& a, const float* priority,
+                                 const int64_t* seg_off_host, int n_seg, double keep_ratio, uint8_t* mask) {
+    if (a.N == 0) return cudaSuccess;
+    k4::Params p;
+    p.values = a.values;
+    p.P = a.P;
+    p.dv = a.dv;
+    p.top_k = a.top_k;
+    p.scene = a.scene;
+    p.prim = a.prim;
+    p.weight = a.weight;
+    p.sel = nullptr;
+    p.N = a.N;
+    p.S = a.S;
+    p.n_layers = a.n_layers;
+    for (int l = 0; l < a.n_layers; ++l) p.hidden[l] = a.hidden[l];
+    k5::Params sp;
+    sp.priority = priority;
+    sp.mask = mask;
+    sp.sel = nullptr;
+    sp.keep_ratio = keep_ratio;
+    sp.n_seg = n_seg;
+    for (int i = 0; i <= n_seg; ++i) sp.off[i] = seg_off_host ? seg_off_host[i] : (i == 0 ? 0 : a.N);
+    const int chunks = a.dv / (a.dtype == LOOKME_BF16 ? 8 : 4);
+    int threads = (chunks + 31) / 32 * 32;
+    if (threads > k4::kThreads) threads = k4::kThreads;
+    if (threads < 128) threads = 128;  // the rank count wants some width too
+    if (a.dtype == LOOKME_BF16)
+        return launch_pdl(k45_select_inject<__nv_bfloat16>, dim3((unsigned)a.N), dim3(threads), 0, c.stream, p, sp);
+    return launch_pdl(k45_select_inject<float>, dim3((unsigned)a.N), dim3(threads), 0, c.stream, p, sp);
 }
 
 cudaError_t launch_inject(const LaunchCtx& c, const InjectArgs& a) {

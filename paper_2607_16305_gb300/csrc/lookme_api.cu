@@ -37,8 +37,9 @@ lookme_status fail(lookme_status st, const char* fmt, ...) {
     return st;
 }
 
-const char* kKernelNames[KID_COUNT] = {"prep",   "route_tc", "route_simt",    "bucket",    "score",       "select",
-                                       "inject", "stage",    "centroid_mean", "inv_cnorm", "route_decode"};
+const char* kKernelNames[KID_COUNT] = {"prep",         "route_tc", "route_simt",    "bucket",
+                                       "score",        "select",   "inject",        "stage",
+                                       "centroid_mean", "inv_cnorm", "route_decode", "select_inject"};
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point, so the
 // library does not link libcuda directly.
@@ -590,9 +591,8 @@ lookme_status lookme_inject(lookme_table* t, const int32_t* scene, const int32_t
     uint8_t* mask = mask_out ? mask_out : t->mask;
     int32_t* sel = sel_out ? sel_out : t->sel;
     const float* pr = priority ? priority : t->qnorm;
-    st = launch(t, s, KID_SELECT, [&] { return launch_select(ctx, pr, N, off.data(), n_seg, keep_ratio, mask, sel); });
-    if (st != LOOKME_OK) return st;
-    if (n_sel == 0) return LOOKME_OK;
+    int64_t max_seg = 0;
+    for (int i = 0; i < n_seg; ++i) max_seg = std::max(max_seg, off[i + 1] - off[i]);
     InjectArgs a;
     a.dtype = d.dtype;
     a.values = t->values;
@@ -608,6 +608,14 @@ lookme_status lookme_inject(lookme_table* t, const int32_t* scene, const int32_t
     a.S = d.n_scenes;
     a.n_layers = n_layers;
     for (int l = 0; l < n_layers; ++l) a.hidden[l] = hidden[l];
+    // Short segments and no kept-id list: selection fused into the injection.
+    if (!sel_out && max_seg <= kFusedMaxSegment)
+        return launch(t, s, KID_SELECT_INJECT, [&] {
+            return launch_select_inject(ctx, a, pr, off.data(), n_seg, keep_ratio, mask);
+        });
+    st = launch(t, s, KID_SELECT, [&] { return launch_select(ctx, pr, N, off.data(), n_seg, keep_ratio, mask, sel); });
+    if (st != LOOKME_OK) return st;
+    if (n_sel == 0) return LOOKME_OK;
     return launch(t, s, KID_INJECT, [&] { return launch_inject(ctx, a); });
 }
 

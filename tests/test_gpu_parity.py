@@ -22,7 +22,10 @@ def _bias(w, scale, seed=11):
 
 
 def run_case(o, lookme_lib, w, *, sample=None, give_centroids=True, bias_scale=0.0, n_layers=None,
-             residency=None, table=0, mu=None, report=None):
+             residency=None, table=0, mu=None, report=None, with_sel=False):
+    """with_sel requests the kept-id list, which routes the injection through
+    the separate selection kernel; without it short segments take the fused
+    select + inject kernel."""
     from paper_2607_16305_gb300 import lookme
 
     L = n_layers or w.layers_per_table
@@ -38,7 +41,7 @@ def run_case(o, lookme_lib, w, *, sample=None, give_centroids=True, bias_scale=0
         qn = torch.empty(N, dtype=torch.float32, device=DEV)
         scene, prim, weight = t.lookup(q, w.top_k, qnorm_out=qn)
         n_sel = sum(int(np.floor((seg_off[i + 1] - seg_off[i]) * w.keep_ratio)) for i in range(len(seg_off) - 1))
-        sel = torch.empty(max(n_sel, 1), dtype=torch.int32, device=DEV)
+        sel = torch.empty(max(n_sel, 1), dtype=torch.int32, device=DEV) if with_sel else None
         mask = t.inject(scene, prim, weight, hs, w.keep_ratio,
                         seg_offsets=seg_off if w.n_segments > 1 else None, sel_out=sel)
         torch.cuda.synchronize()
@@ -72,7 +75,7 @@ def run_case(o, lookme_lib, w, *, sample=None, give_centroids=True, bias_scale=0
     assert np.abs(qn.cpu().numpy() - qn_all).max() <= 1e-4 * max(1.0, qn_all.max())
     gmask = mask.cpu().numpy()
     mask_ties = H.check_mask(o, qn_all, gmask, w.keep_ratio, seg_off)
-    if n_sel:
+    if n_sel and with_sel:
         H.check_sel(sel[:n_sel].cpu().numpy(), gmask, w.keep_ratio, seg_off)
 
     # ---- hidden: untouched rows bit-identical, kept rows against the oracle
@@ -103,8 +106,9 @@ def test_tiny_fp32_full(oracle, lookme_lib):
     run_case(oracle, lookme_lib, W.WORKLOADS["tiny_fp32"])
 
 
-def test_single_image_full(oracle, lookme_lib):
-    res = run_case(oracle, lookme_lib, W.WORKLOADS["single_image"])
+@pytest.mark.parametrize("with_sel", [False, True], ids=["fused_select", "select_list"])
+def test_single_image_full(oracle, lookme_lib, with_sel):
+    res = run_case(oracle, lookme_lib, W.WORKLOADS["single_image"], with_sel=with_sel)
     assert res["scene_ties"] == 0
 
 
@@ -113,6 +117,7 @@ def test_batched_zipf_sampled(oracle, lookme_lib):
     w = W.WORKLOADS["batched_zipf"]
     rng = np.random.default_rng(0)
     run_case(oracle, lookme_lib, w, sample=rng.choice(w.n_tokens, 512, replace=False))
+    run_case(oracle, lookme_lib, w, sample=rng.choice(w.n_tokens, 256, replace=False), with_sel=True)
 
 
 @pytest.mark.slow
@@ -151,7 +156,7 @@ SMALL_CASES = [
 @pytest.mark.parametrize("name,kw", SMALL_CASES, ids=[c[0] for c in SMALL_CASES])
 def test_small_shapes(oracle, lookme_lib, dtype, name, kw):
     w = W.small(f"{name}_{dtype}", dtype=dtype, **kw)
-    run_case(oracle, lookme_lib, w)
+    run_case(oracle, lookme_lib, w, with_sel=(name in ("s2", "s6", "s8")))
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "fp32"])
