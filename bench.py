@@ -7,8 +7,11 @@ add) over one batch of seeded synthetic tokens: the single-image workload
 keep 25%) unless --workload says otherwise.
 
   value      tokens/s over K device-timed steps (CUDA events on the launching
-             stream, L2 flushed by a 512 MiB write before every step, outside
-             the events), inputs resident in HBM
+             stream; the step replayed as one CUDA graph of the library's
+             kernels; L2 flushed by writing then reading 512 MiB before every
+             step, outside the events), inputs resident in HBM.  The eager
+             time (the same calls issued one by one from Python) is reported
+             beside it.
   e2e        the same through host buffers: pinned-host queries and hidden
              states copied in and the updated hidden states copied out, inside
              the timed region
@@ -71,7 +74,7 @@ def load_peaks():
 
 def kernel_source_sha():
     h = hashlib.sha256()
-    with open(os.path.join(ROOT, "paper_2607_16305_gb300", "csrc", "k_score.cu"), "rb") as f:
+    with open(os.path.join(ROOT, "paper_2607_16305_gb300", "csrc", "k_score_tc.cu"), "rb") as f:
         h.update(f.read())
     return h.hexdigest()[:16]
 
@@ -178,17 +181,41 @@ def run_lookme(args, w, ws, rank, local):
     mask = torch.empty(N, dtype=torch.uint8, device=dev)
     seg = w.segment_offsets if w.n_segments > 1 else None
     flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
+    flush_sink = torch.zeros((), dtype=torch.int64, device=dev)
 
     def step():
         t.lookup(q, K, scene, prim, weight)
         t.inject(scene, prim, weight, hidden, w.keep_ratio, seg_offsets=seg, mask_out=mask)
 
+    def flush_l2(i):
+        # Write then read a buffer four times L2's size: the step starts with no
+        # table data in L2 and no dirty flush lines left to write back.
+        flush.fill_(i & 0xFF)
+        flush_sink.copy_(flush.sum(dtype=torch.int64))
+
     for _ in range(args.warmup):
-        flush.fill_(1)
+        flush_l2(1)
         step()
     torch.cuda.synchronize(dev)
     stats = t.stats()
     n_sel = int(mask.sum().item())
+
+    # The step as one CUDA graph (the library never allocates or syncs inside a
+    # call once scratch is reserved), replayed per timed step.
+    graph = torch.cuda.CUDAGraph()
+    side = torch.cuda.Stream(dev)
+    side.wait_stream(stream)
+    with torch.cuda.stream(side):
+        step()
+    stream.wait_stream(side)
+    with torch.cuda.graph(graph):
+        step()
+    torch.cuda.synchronize(dev)
+
+    c0 = t.launch_count()
+    step()
+    torch.cuda.synchronize(dev)
+    launches_per_step = t.launch_count() - c0
 
     sampler = ClockSampler(local)
     sampler.start()
@@ -200,18 +227,28 @@ def run_lookme(args, w, ws, rank, local):
 
         dist.barrier()
     torch.cuda.synchronize(dev)
-    launches0 = t.launch_count()
     for i in range(args.steps):
-        flush.fill_(i & 0xFF)
+        flush_l2(i)
         starts[i].record(stream)
-        step()
+        graph.replay()
         ends[i].record(stream)
     torch.cuda.synchronize(dev)
-    launches = t.launch_count() - launches0
     if ws > 1:
         dist.barrier()
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     total_ms = sum(step_ms)
+    launches = launches_per_step * args.steps
+
+    # ------------------------------------ the same steps as eager C-ABI calls
+    estarts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    eends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    for i in range(args.steps):
+        flush_l2(i)
+        estarts[i].record(stream)
+        step()
+        eends[i].record(stream)
+    torch.cuda.synchronize(dev)
+    eager_ms = sum(s.elapsed_time(e) for s, e in zip(estarts, eends)) / args.steps
 
     # ----------------------------------------- per-kernel durations (traced)
     t.trace_enable(True)
@@ -219,7 +256,7 @@ def run_lookme(args, w, ws, rank, local):
     tstarts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     tends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     for i in range(args.steps):
-        flush.fill_(i & 0xFF)
+        flush_l2(i)
         tstarts[i].record(stream)
         step()
         tends[i].record(stream)
@@ -241,7 +278,7 @@ def run_lookme(args, w, ws, rank, local):
     e_starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     e_ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     for i in range(args.steps):
-        flush.fill_(i & 0xFF)
+        flush_l2(i)
         e_starts[i].record(stream)
         q_dev.copy_(q_host, non_blocking=True)
         for hd, hh in zip(h_dev, h_host):
@@ -281,7 +318,8 @@ def run_lookme(args, w, ws, rank, local):
         "vs_baseline": None, "dtype": w.dtype, "data": "synthetic (seeded Gaussian mixture, random tables)",
         "config": {"workload": w.name, "tokens": N, "d_key": w.d_key, "scenes": w.n_scenes, "prims": w.n_prims,
                    "d_value": w.d_value, "top_k": K, "keep_ratio": w.keep_ratio, "layers": w.layers_per_table,
-                   "l2": f"flushed before every step ({FLUSH_BYTES >> 20} MiB write, outside the events)",
+                   "l2": f"flushed before every step ({FLUSH_BYTES >> 20} MiB written then read, outside the events)",
+                   "launch": "step replayed as one CUDA graph (kernels chained by programmatic dependent launch)",
                    "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "kernel": "score (level-2 key scoring + top-k + softmax)",
                      "achieved": achieved, "peak": hbm, "unit": "GB/s",
@@ -290,6 +328,7 @@ def run_lookme(args, w, ws, rank, local):
                      "traffic": profiled_traffic(w.name)},
         "step_roofline": {"bound": "hbm", "algorithmic_bytes": ab["step"], "achieved": step_gbs, "peak": hbm,
                           "unit": "GB/s", "frac": step_gbs / hbm, "roofline_us": ab["step"] / hbm / 1e3},
+        "eager_ms_per_step": eager_ms,
         "kernels_ms": kernels_ms, "traced_ms_per_step": traced_ms / args.steps,
         "routed_scenes": stats["n_routed_scenes"], "selected_tokens": n_sel,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,

@@ -130,18 +130,20 @@ struct LaunchCtx {
 cudaError_t launch_prep(const LaunchCtx& c, int dtype, const void* q, int64_t N, int dk, float* qnorm,
                         float* qnorm_out, unsigned long long* best);
 // K1 (tcgen05, bf16, d_k <= 512).  tmap_q is the CUtensorMap of the queries
-// (box 64 x 128); tmap_c[i] the centroids' map with box 64 x (64 << i).
+// (box 64 x 128); tmap_c[i] the centroids' map with box 64 x (64 << i).  Also
+// computes ||q|| into qnorm (and qnorm_out if given), so no prep kernel runs;
+// every key of best[0, N) must be 0 on entry.
 constexpr int kRouteTcMaxDk = 512;
 cudaError_t launch_route_tc(const LaunchCtx& c, const void* tmap_q, const void* const tmap_c[3], int64_t N,
-                            int64_t S, int dk, const float* inv_cnorm, const float* bias, const float* qnorm,
-                            unsigned long long* best, uint32_t* status);
+                            int64_t S, int dk, const float* inv_cnorm, const float* bias, float* qnorm,
+                            float* qnorm_out, unsigned long long* best, uint32_t* status);
 // K1 (CUDA cores)
 cudaError_t launch_route_simt(const LaunchCtx& c, int dtype, const void* q, const void* cent, int64_t N,
                               int64_t S, int dk, const float* inv_cnorm, const float* bias, const float* qnorm,
                               unsigned long long* best);
-// K2
+// K2 (also resets best[0, N) to 0 for the next call)
 constexpr int kTokensPerItem = 8;
-cudaError_t launch_bucket(const LaunchCtx& c, const unsigned long long* best, int64_t N, int64_t S,
+cudaError_t launch_bucket(const LaunchCtx& c, unsigned long long* best, int64_t N, int64_t S,
                           int32_t* scene_out, int32_t* perm, WorkItem* work, int32_t* routed, int32_t* counters);
 // K3
 struct ScoreArgs {

@@ -61,7 +61,7 @@ __device__ void block_exclusive_scan3(int3 v, int3& excl, int3& total, int3* war
 }  // namespace
 
 __global__ void __launch_bounds__(kThreads, 1)
-    k2_bucket(const unsigned long long* __restrict__ best, int64_t N, int S, int32_t* __restrict__ scene_out,
+    k2_bucket(unsigned long long* __restrict__ best, int64_t N, int S, int32_t* __restrict__ scene_out,
               int32_t* __restrict__ perm, WorkItem* __restrict__ work, int32_t* __restrict__ routed,
               int32_t* __restrict__ counters) {
     extern __shared__ int cnt[];  // [S]: counts, then running token offsets
@@ -123,12 +123,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int64_t t = tid; t < N; t += kThreads) {
         const int32_t s = unpack_scene(best[t], S);
+        best[t] = 0ull;  // ready for the next call's argmax
         const int pos = atomicAdd(&cnt[s], 1);
         perm[pos] = (int32_t)t;
     }
 }
 
-cudaError_t launch_bucket(const LaunchCtx& c, const unsigned long long* best, int64_t N, int64_t S,
+cudaError_t launch_bucket(const LaunchCtx& c, unsigned long long* best, int64_t N, int64_t S,
                           int32_t* scene_out, int32_t* perm, WorkItem* work, int32_t* routed, int32_t* counters) {
     const size_t smem = (size_t)S * sizeof(int);
     return launch_pdl(k2_bucket, dim3(1), dim3(kThreads), smem, c.stream, best, N, (int)S, scene_out, perm, work,

@@ -179,20 +179,24 @@ struct Params {
 };
 }  // namespace k4
 
-// Gather + weighted sum + residual add for token t by one CTA.
+// Row pointers and weights of token t's k value rows, in shared memory.
 template <typename T>
-__device__ __forceinline__ void inject_token(const k4::Params& p, int64_t t) {
-    constexpr int EPC = Vec16<T>::N;
-    constexpr int BATCH = 8;  // value rows in flight per thread
-    __shared__ const uint4* rows[LOOKME_MAX_TOP_K];
-    __shared__ float w[LOOKME_MAX_TOP_K];
+__device__ __forceinline__ void load_rows(const k4::Params& p, int64_t t, const uint4** rows, float* w) {
     const int64_t s = min(max((int64_t)p.scene[t], (int64_t)0), p.S - 1);
     for (int j = threadIdx.x; j < p.top_k; j += blockDim.x) {
         const int64_t pr = min(max((int64_t)p.prim[t * p.top_k + j], (int64_t)0), p.P - 1);
         rows[j] = reinterpret_cast<const uint4*>(reinterpret_cast<const T*>(p.values) + (s * p.P + pr) * p.dv);
         w[j] = p.weight[t * p.top_k + j];
     }
-    __syncthreads();
+}
+
+// Weighted sum of the k rows (fp32) added into token t's row of every layer,
+// one rounding; the CTA's threads stride over 16-byte chunks of the row.
+template <typename T>
+__device__ __forceinline__ void accumulate_store(const k4::Params& p, int64_t t, const uint4* const* rows,
+                                                 const float* w) {
+    constexpr int EPC = Vec16<T>::N;
+    constexpr int BATCH = 8;  // value rows in flight per thread
     const int chunks = p.dv / EPC;
     for (int ch = threadIdx.x; ch < chunks; ch += blockDim.x) {
         uint4* h0 = reinterpret_cast<uint4*>(reinterpret_cast<T*>(p.hidden[0]) + t * p.dv) + ch;
@@ -229,9 +233,14 @@ __device__ __forceinline__ void inject_token(const k4::Params& p, int64_t t) {
 
 template <typename T>
 __global__ void __launch_bounds__(k4::kThreads) k4_inject(const __grid_constant__ k4::Params p) {
+    __shared__ const uint4* rows[LOOKME_MAX_TOP_K];
+    __shared__ float w[LOOKME_MAX_TOP_K];
     pdl_trigger();
     pdl_wait();
-    inject_token<T>(p, p.sel[blockIdx.x]);
+    const int64_t t = p.sel[blockIdx.x];
+    load_rows<T>(p, t, rows, w);
+    __syncthreads();
+    accumulate_store<T>(p, t, rows, w);
 }
 
 // Selection fused into the injection (segments of at most kFusedMaxSegment
@@ -239,14 +248,18 @@ __global__ void __launch_bounds__(k4::kThreads) k4_inject(const __grid_constant_
 //   rank_t = #{ j : pi_j > pi_t, or pi_j == pi_t and j < t },
 // which orders tokens exactly like the radix selection (larger priority
 // first, lower index on ties); the token is kept iff rank_t < r.  Kept tokens
-// are injected by the same CTA.
+// are injected by the same CTA.  The token's value-row addresses are loaded
+// before the rank is known, so the two dependent loads overlap.
 template <typename T>
 __global__ void __launch_bounds__(k4::kThreads) k45_select_inject(const __grid_constant__ k4::Params p,
                                                                   const __grid_constant__ k5::Params sp) {
     __shared__ int warp_cnt[k4::kThreads / 32];
+    __shared__ const uint4* rows[LOOKME_MAX_TOP_K];
+    __shared__ float w[LOOKME_MAX_TOP_K];
     pdl_trigger();
     pdl_wait();
     const int64_t t = blockIdx.x;
+    load_rows<T>(p, t, rows, w);
     int lo = 0, hi = sp.n_seg;  // segment: off[lo] <= t < off[lo + 1]
     while (hi - lo > 1) {
         const int mid = (lo + hi) / 2;
@@ -272,7 +285,10 @@ __global__ void __launch_bounds__(k4::kThreads) k45_select_inject(const __grid_c
         keep = total < r;
     }
     if (threadIdx.x == 0 && sp.mask) sp.mask[t] = (uint8_t)keep;
-    if (keep) inject_token<T>(p, t);
+    if (keep) {
+        __syncthreads();  // row addresses visible to every thread
+        accumulate_store<T>(p, t, rows, w);
+    }
 }
 
 cudaError_t launch_select_inject(const LaunchCtx& c, const InjectArgs& a, const float* priority,
@@ -298,10 +314,9 @@ cudaError_t launch_select_inject(const LaunchCtx& c, const InjectArgs& a, const 
     sp.keep_ratio = keep_ratio;
     sp.n_seg = n_seg;
     for (int i = 0; i <= n_seg; ++i) sp.off[i] = seg_off_host ? seg_off_host[i] : (i == 0 ? 0 : a.N);
-    const int chunks = a.dv / (a.dtype == LOOKME_BF16 ? 8 : 4);
-    int threads = (chunks + 31) / 32 * 32;
-    if (threads > k4::kThreads) threads = k4::kThreads;
-    if (threads < 128) threads = 128;  // the rank count wants some width too
+    // 128 threads: every CTA of a 1,024-token call is resident at once, and a
+    // 2,048-wide row is two 16-byte chunks per thread.
+    const int threads = 128;
     if (a.dtype == LOOKME_BF16)
         return launch_pdl(k45_select_inject<__nv_bfloat16>, dim3((unsigned)a.N), dim3(threads), 0, c.stream, p, sp);
     return launch_pdl(k45_select_inject<float>, dim3((unsigned)a.N), dim3(threads), 0, c.stream, p, sp);

@@ -170,7 +170,7 @@ template <int BN, int STAGES>
 __global__ void __launch_bounds__(k1tc::kThreads, 1)
     k1_route_tc(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_c,
                 int64_t N, int64_t S, int dk, int tiles_per_cta, const float* __restrict__ inv_cnorm,
-                const float* __restrict__ bias, const float* __restrict__ qnorm,
+                const float* __restrict__ bias, float* __restrict__ qnorm, float* __restrict__ qnorm_out,
                 unsigned long long* __restrict__ best, uint32_t* __restrict__ status) {
     using namespace k1tc;
     extern __shared__ uint8_t smem_raw[];
@@ -285,10 +285,33 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
         // Epilogue warps 2..5 own TMEM lane quarters (warp % 4) * 32 .. + 31.
         const int quarter = warp & 3;
         const int64_t row = (int64_t)m_tile * BM + quarter * 32 + lane;
+        // ||q_row||_2 from the token tile in shared memory: every 16-byte chunk
+        // of the row is read once (lane-rotated to avoid bank conflicts; the
+        // swizzle only permutes chunks within the row, and zero-filled columns
+        // past d_k add nothing).
         float inv_q = 1.f;
-        if (bias && row < N) {
-            const float n = qnorm[row];
-            inv_q = n > 0.f ? 1.f / n : 0.f;
+        if (blockIdx.y == 0 || bias) {
+            const bool ready = ptx::mbar_wait(a_full, 0, abort, kTimeoutNs);
+            float ss = 0.f;
+            if (ready) {
+                const int r = quarter * 32 + lane;
+                for (int kb = 0; kb < nkb; ++kb) {
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        float f[8];
+                        Vec16<__nv_bfloat16>::unpack(
+                            *reinterpret_cast<const uint4*>(sA + kb * BM * 128 + r * 128 + (((c + lane) & 7) * 16)), f);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) ss = fmaf(f[i], f[i], ss);
+                    }
+                }
+            }
+            const float n = sqrtf(ss);
+            if (blockIdx.y == 0 && row < N && ready) {
+                qnorm[row] = n;
+                if (qnorm_out) qnorm_out[row] = n;
+            }
+            if (bias) inv_q = n > 0.f ? 1.f / n : 0.f;
         }
         unsigned long long key = 0ull;
         for (int it = 0, nt = nt0; nt < nt1; ++nt, ++it) {
@@ -349,8 +372,8 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
 
 template <int BN, int STAGES>
 static cudaError_t launch_route_tc_t(const LaunchCtx& c, const void* tmap_q, const void* tmap_c, int64_t N,
-                                     int64_t S, int dk, const float* inv_cnorm, const float* bias,
-                                     const float* qnorm, unsigned long long* best, uint32_t* status) {
+                                     int64_t S, int dk, const float* inv_cnorm, const float* bias, float* qnorm,
+                                     float* qnorm_out, unsigned long long* best, uint32_t* status) {
     using namespace k1tc;
     const int nkb = (dk + BK - 1) / BK;
     // Keep TMEM demand per SM within its 512 columns: at most 512 / (2 BN)
@@ -372,21 +395,24 @@ static cudaError_t launch_route_tc_t(const LaunchCtx& c, const void* tmap_q, con
     memcpy(&mq, tmap_q, sizeof(CUtensorMap));
     memcpy(&mc, tmap_c, sizeof(CUtensorMap));
     return launch_pdl(k1_route_tc<BN, STAGES>, dim3(m_tiles, splits), dim3(kThreads), (size_t)smem, c.stream, mq, mc,
-                      N, S, dk, per, inv_cnorm, bias, qnorm, best, status);
+                      N, S, dk, per, inv_cnorm, bias, qnorm, qnorm_out, best, status);
 }
 
 cudaError_t launch_route_tc(const LaunchCtx& c, const void* tmap_q, const void* const tmap_c[3], int64_t N,
-                            int64_t S, int dk, const float* inv_cnorm, const float* bias, const float* qnorm,
-                            unsigned long long* best, uint32_t* status) {
+                            int64_t S, int dk, const float* inv_cnorm, const float* bias, float* qnorm,
+                            float* qnorm_out, unsigned long long* best, uint32_t* status) {
     if (N == 0) return cudaSuccess;
     if (dk > kRouteTcMaxDk) return cudaErrorInvalidValue;
     const int m_tiles = (int)((N + k1tc::BM - 1) / k1tc::BM);
     // Narrow scene tiles when there are few token tiles, so more CTAs share the work.
     if ((int64_t)m_tiles * ((S + 255) / 256) >= c.num_sms)
-        return launch_route_tc_t<256, 3>(c, tmap_q, tmap_c[2], N, S, dk, inv_cnorm, bias, qnorm, best, status);
+        return launch_route_tc_t<256, 3>(c, tmap_q, tmap_c[2], N, S, dk, inv_cnorm, bias, qnorm, qnorm_out, best,
+                                          status);
     if ((int64_t)m_tiles * ((S + 127) / 128) >= c.num_sms)
-        return launch_route_tc_t<128, 4>(c, tmap_q, tmap_c[1], N, S, dk, inv_cnorm, bias, qnorm, best, status);
-    return launch_route_tc_t<64, 4>(c, tmap_q, tmap_c[0], N, S, dk, inv_cnorm, bias, qnorm, best, status);
+        return launch_route_tc_t<128, 4>(c, tmap_q, tmap_c[1], N, S, dk, inv_cnorm, bias, qnorm, qnorm_out, best,
+                                          status);
+    return launch_route_tc_t<64, 4>(c, tmap_q, tmap_c[0], N, S, dk, inv_cnorm, bias, qnorm, qnorm_out, best,
+                                          status);
 }
 
 cudaError_t configure_route_kernels() {

@@ -496,17 +496,22 @@ lookme_status lookme_lookup(lookme_table* t, const void* queries, int64_t N, int
     const int dk = (int)d.d_key;
     const float* bias = t->has_bias ? t->bias : nullptr;
 
-    st = launch(t, s, KID_PREP, [&] { return launch_prep(ctx, d.dtype, queries, N, dk, t->qnorm, qnorm_out, t->best); });
-    if (st != LOOKME_OK) return st;
     if (t->tc_route) {
+        // The tcgen05 routing kernel computes the query norms itself; the
+        // argmax keys were reset by the previous call's bucketing (or are
+        // fresh zeroed scratch).
         CUtensorMap mq;
         if (!encode_bf16_2d(&mq, queries, N, dk, 128))
             return fail(LOOKME_ERR_CUDA, "cuTensorMapEncodeTiled failed for the queries");
         const void* mc[3] = {&t->tmap_c[0], &t->tmap_c[1], &t->tmap_c[2]};
         st = launch(t, s, KID_ROUTE_TC, [&] {
-            return launch_route_tc(ctx, &mq, mc, N, d.n_scenes, dk, t->inv_cnorm, bias, t->qnorm, t->best, t->status);
+            return launch_route_tc(ctx, &mq, mc, N, d.n_scenes, dk, t->inv_cnorm, bias, t->qnorm, qnorm_out, t->best,
+                                   t->status);
         });
     } else {
+        st = launch(t, s, KID_PREP,
+                    [&] { return launch_prep(ctx, d.dtype, queries, N, dk, t->qnorm, qnorm_out, t->best); });
+        if (st != LOOKME_OK) return st;
         st = launch(t, s, KID_ROUTE_SIMT, [&] {
             return launch_route_simt(ctx, d.dtype, queries, t->cent, N, d.n_scenes, dk, t->inv_cnorm, bias, t->qnorm,
                                      t->best);
@@ -768,7 +773,8 @@ extern "C" lookme_status lookme_route_scenes_static(lookme_table* t, const void*
             return fail(LOOKME_ERR_CUDA, "cuTensorMapEncodeTiled failed for the queries");
         const void* mc[3] = {&t->tmap_c[0], &t->tmap_c[1], &t->tmap_c[2]};
         st = launch(t, s, KID_ROUTE_TC, [&] {
-            return launch_route_tc(ctx, &mq, mc, N, d.n_scenes, dk, t->inv_cnorm, bias, sc.qnorm, sc.best, t->status);
+            return launch_route_tc(ctx, &mq, mc, N, d.n_scenes, dk, t->inv_cnorm, bias, sc.qnorm, nullptr, sc.best,
+                                   t->status);
         });
     } else {
         st = launch(t, s, KID_ROUTE_SIMT, [&] {
