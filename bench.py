@@ -1,8 +1,9 @@
 """Benchmark of the LookME lookup + sparse injection on GB300.
 
-A step is one lookme_lookup + lookme_inject pair (level-1 routing, bucketing,
-level-2 scoring with top-k and softmax, token selection, gather and residual
-add) over one batch of seeded synthetic tokens: the single-image workload
+A step is one lookme_lookup_inject call (level-1 routing, bucketing, level-2
+scoring with top-k and softmax, token selection, gather and residual add; the
+same results as lookme_lookup + lookme_inject) over one batch of seeded
+synthetic tokens: the single-image workload
 (1,024 tokens, d_k 256, 1,024 scenes x 256 primitives, d_v 2,048, bf16, top-8,
 keep 25%) unless --workload says otherwise.
 
@@ -184,8 +185,8 @@ def run_lookme(args, w, ws, rank, local):
     flush_sink = torch.zeros((), dtype=torch.int64, device=dev)
 
     def step():
-        t.lookup(q, K, scene, prim, weight)
-        t.inject(scene, prim, weight, hidden, w.keep_ratio, seg_offsets=seg, mask_out=mask)
+        t.lookup_inject(q, K, hidden, w.keep_ratio, seg_offsets=seg, scene_out=scene, prim_out=prim,
+                        weight_out=weight, mask_out=mask)
 
     def flush_l2(i):
         # Write then read a buffer four times L2's size: the step starts with no
@@ -283,8 +284,8 @@ def run_lookme(args, w, ws, rank, local):
         q_dev.copy_(q_host, non_blocking=True)
         for hd, hh in zip(h_dev, h_host):
             hd.copy_(hh, non_blocking=True)
-        t.lookup(q_dev, K, scene, prim, weight)
-        t.inject(scene, prim, weight, h_dev, w.keep_ratio, seg_offsets=seg, mask_out=mask)
+        t.lookup_inject(q_dev, K, h_dev, w.keep_ratio, seg_offsets=seg, scene_out=scene, prim_out=prim,
+                        weight_out=weight, mask_out=mask)
         for ho, hd in zip(h_out, h_dev):
             ho.copy_(hd, non_blocking=True)
         e_ends[i].record(stream)

@@ -161,6 +161,17 @@ lookme_status lookme_inject(lookme_table* table, const int32_t* scene, const int
                             double keep_ratio, void* const* hidden, int32_t n_layers,
                             uint8_t* mask_out, int32_t* sel_out, lookme_stream stream);
 
+/* lookme_lookup followed by lookme_inject in one call, on one stream, with
+ * the same results (Sec. "Hierarchical Lookup" then Sec. "Sparse Injection").
+ * The arguments mean what they mean there; priority NULL = the query norms of
+ * these queries; mask_out (device [n_tokens] uint8, or NULL) receives the
+ * gate.  Errors: those of lookme_lookup, then those of lookme_inject (the
+ * lookup's outputs are written when only the injection fails). */
+lookme_status lookme_lookup_inject(lookme_table* table, const void* queries, int64_t n_tokens, int32_t top_k,
+                                   const float* priority, const int64_t* seg_offsets, int32_t n_seg,
+                                   double keep_ratio, void* const* hidden, int32_t n_layers, int32_t* scene_out,
+                                   int32_t* prim_out, float* weight_out, uint8_t* mask_out, lookme_stream stream);
+
 /* Size the per-call scratch for up to max_tokens tokens now, so that later
  * calls (for example under CUDA graph capture) never allocate.  Synchronous. */
 lookme_status lookme_reserve(lookme_table* table, int64_t max_tokens);

@@ -248,18 +248,24 @@ __global__ void __launch_bounds__(k4::kThreads) k4_inject(const __grid_constant_
 //   rank_t = #{ j : pi_j > pi_t, or pi_j == pi_t and j < t },
 // which orders tokens exactly like the radix selection (larger priority
 // first, lower index on ties); the token is kept iff rank_t < r.  Kept tokens
-// are injected by the same CTA.  The token's value-row addresses are loaded
-// before the rank is known, so the two dependent loads overlap.
+// are injected by the same CTA.  Every load the rank and the row addresses
+// need is issued before any is used, so the kernel costs one L2 round trip
+// for the gate and one HBM round trip for the injection.
+namespace k45 {
+constexpr int kThreads = 256;  // one 16-byte chunk of a 2,048-wide bf16 row per thread
+constexpr int kUnroll = 4;     // priorities in flight per thread and pass
+}  // namespace k45
+
 template <typename T>
-__global__ void __launch_bounds__(k4::kThreads) k45_select_inject(const __grid_constant__ k4::Params p,
-                                                                  const __grid_constant__ k5::Params sp) {
-    __shared__ int warp_cnt[k4::kThreads / 32];
+__global__ void __launch_bounds__(k45::kThreads) k45_select_inject(const __grid_constant__ k4::Params p,
+                                                                   const __grid_constant__ k5::Params sp) {
+    __shared__ int warp_cnt[k45::kThreads / 32];
     __shared__ const uint4* rows[LOOKME_MAX_TOP_K];
     __shared__ float w[LOOKME_MAX_TOP_K];
     pdl_trigger();
     pdl_wait();
     const int64_t t = blockIdx.x;
-    load_rows<T>(p, t, rows, w);
+    const int tid = threadIdx.x;
     int lo = 0, hi = sp.n_seg;  // segment: off[lo] <= t < off[lo + 1]
     while (hi - lo > 1) {
         const int mid = (lo + hi) / 2;
@@ -268,27 +274,58 @@ __global__ void __launch_bounds__(k4::kThreads) k45_select_inject(const __grid_c
     }
     const int64_t b = sp.off[lo], len = sp.off[lo + 1] - b;
     const int64_t r = (int64_t)floor((double)len * sp.keep_ratio);
-    bool keep = r >= len;
-    if (r > 0 && r < len) {
+    if (r <= 0) {
+        if (tid == 0 && sp.mask) sp.mask[t] = 0;
+        return;
+    }
+    // Row addresses and weights (threads < top_k) and the first pass of
+    // priorities are independent loads, in flight together.
+    int32_t sc = 0, pj = 0;
+    float wj = 0.f;
+    if (tid < p.top_k) {
+        sc = p.scene[t];
+        pj = p.prim[t * p.top_k + tid];
+        wj = p.weight[t * p.top_k + tid];
+    }
+    bool keep = true;
+    if (r < len) {
+        const float* pb = sp.priority + b;
         const uint32_t kt = k5::prio_key(sp.priority[t]);
+        const int64_t tl = t - b;
         int cnt = 0;
-        for (int64_t j = threadIdx.x; j < len; j += blockDim.x) {
-            const uint32_t kj = k5::prio_key(sp.priority[b + j]);
-            cnt += (kj > kt) || (kj == kt && b + j < t);
+        for (int64_t j0 = tid; j0 < len; j0 += k45::kUnroll * k45::kThreads) {
+            float v[k45::kUnroll];
+#pragma unroll
+            for (int u = 0; u < k45::kUnroll; ++u) {
+                const int64_t j = j0 + u * k45::kThreads;
+                v[u] = j < len ? pb[j] : 0.f;
+            }
+#pragma unroll
+            for (int u = 0; u < k45::kUnroll; ++u) {
+                const int64_t j = j0 + u * k45::kThreads;
+                const uint32_t kj = k5::prio_key(v[u]);
+                cnt += j < len && ((kj > kt) || (kj == kt && j < tl));
+            }
         }
 #pragma unroll
         for (int o = 16; o; o >>= 1) cnt += __shfl_xor_sync(0xFFFFFFFFu, cnt, o);
-        if ((threadIdx.x & 31) == 0) warp_cnt[threadIdx.x / 32] = cnt;
-        __syncthreads();
+        if ((tid & 31) == 0) warp_cnt[tid / 32] = cnt;
+    }
+    if (tid < p.top_k) {
+        const int64_t s = min(max((int64_t)sc, (int64_t)0), p.S - 1);
+        const int64_t pr = min(max((int64_t)pj, (int64_t)0), p.P - 1);
+        rows[tid] = reinterpret_cast<const uint4*>(reinterpret_cast<const T*>(p.values) + (s * p.P + pr) * p.dv);
+        w[tid] = wj;
+    }
+    __syncthreads();  // counts, row addresses and weights visible to every thread
+    if (r < len) {
         int total = 0;
-        for (int i = 0; i < (int)(blockDim.x / 32); ++i) total += warp_cnt[i];
+#pragma unroll
+        for (int i = 0; i < k45::kThreads / 32; ++i) total += warp_cnt[i];
         keep = total < r;
     }
-    if (threadIdx.x == 0 && sp.mask) sp.mask[t] = (uint8_t)keep;
-    if (keep) {
-        __syncthreads();  // row addresses visible to every thread
-        accumulate_store<T>(p, t, rows, w);
-    }
+    if (tid == 0 && sp.mask) sp.mask[t] = (uint8_t)keep;
+    if (keep) accumulate_store<T>(p, t, rows, w);
 }
 
 cudaError_t launch_select_inject(const LaunchCtx& c, const InjectArgs& a, const float* priority,
@@ -314,12 +351,10 @@ cudaError_t launch_select_inject(const LaunchCtx& c, const InjectArgs& a, const 
     sp.keep_ratio = keep_ratio;
     sp.n_seg = n_seg;
     for (int i = 0; i <= n_seg; ++i) sp.off[i] = seg_off_host ? seg_off_host[i] : (i == 0 ? 0 : a.N);
-    // 128 threads: every CTA of a 1,024-token call is resident at once, and a
-    // 2,048-wide row is two 16-byte chunks per thread.
-    const int threads = 128;
     if (a.dtype == LOOKME_BF16)
-        return launch_pdl(k45_select_inject<__nv_bfloat16>, dim3((unsigned)a.N), dim3(threads), 0, c.stream, p, sp);
-    return launch_pdl(k45_select_inject<float>, dim3((unsigned)a.N), dim3(threads), 0, c.stream, p, sp);
+        return launch_pdl(k45_select_inject<__nv_bfloat16>, dim3((unsigned)a.N), dim3(k45::kThreads), 0, c.stream,
+                          p, sp);
+    return launch_pdl(k45_select_inject<float>, dim3((unsigned)a.N), dim3(k45::kThreads), 0, c.stream, p, sp);
 }
 
 cudaError_t launch_inject(const LaunchCtx& c, const InjectArgs& a) {

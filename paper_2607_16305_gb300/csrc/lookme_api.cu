@@ -624,6 +624,18 @@ lookme_status lookme_inject(lookme_table* t, const int32_t* scene, const int32_t
     return launch(t, s, KID_INJECT, [&] { return launch_inject(ctx, a); });
 }
 
+lookme_status lookme_lookup_inject(lookme_table* t, const void* queries, int64_t N, int32_t top_k,
+                                   const float* priority, const int64_t* seg_offsets, int32_t n_seg,
+                                   double keep_ratio, void* const* hidden, int32_t n_layers, int32_t* scene_out,
+                                   int32_t* prim_out, float* weight_out, uint8_t* mask_out, lookme_stream stream) {
+    // The lookup's outputs feed the injection on the same stream; with PDL the
+    // injection kernel's launch overlaps the tail of the level-2 kernel.
+    lookme_status st = lookme_lookup(t, queries, N, top_k, scene_out, prim_out, weight_out, nullptr, stream);
+    if (st != LOOKME_OK) return st;
+    return lookme_inject(t, scene_out, prim_out, weight_out, N, top_k, priority, seg_offsets, n_seg, keep_ratio,
+                         hidden, n_layers, mask_out, nullptr, stream);
+}
+
 lookme_status lookme_last_lookup_stats(lookme_table* t, lookme_lookup_stats* out, lookme_stream stream) {
     lookme_status st = check_table(t);
     if (st != LOOKME_OK) return st;

@@ -26,7 +26,7 @@ EXPORTS = [
     "lookme_table_create", "lookme_table_destroy", "lookme_load_scenes", "lookme_lookup", "lookme_inject",
     "lookme_reserve", "lookme_last_lookup_stats", "lookme_device_status", "lookme_launch_count",
     "lookme_trace_enable", "lookme_trace_read", "lookme_kernel_name", "lookme_status_string",
-    "lookme_last_error", "lookme_route_scenes_static",
+    "lookme_last_error", "lookme_route_scenes_static", "lookme_lookup_inject",
 ]
 
 
@@ -82,6 +82,7 @@ def load(path: str = LIB_PATH):
         "lookme_status_string": ([I32], ctypes.c_char_p),
         "lookme_last_error": ([], ctypes.c_char_p),
         "lookme_route_scenes_static": ([P, P, I64, P, P], I32),
+        "lookme_lookup_inject": ([P, P, I64, I32, P, P, I32, D, P, I32, P, P, P, P, P], I32),
     }
     for name, (argtypes, restype) in sig.items():
         fn = getattr(lib, name)
@@ -205,6 +206,30 @@ class Table:
                                       _ptr(priority), seg, n_seg, float(keep_ratio), arr, len(hidden),
                                       _ptr(mask_out), _ptr(sel_out), _stream(stream, self.device)))
         return mask_out
+
+    def lookup_inject(self, queries, top_k, hidden, keep_ratio, priority=None, seg_offsets=None, scene_out=None,
+                      prim_out=None, weight_out=None, mask_out=None, stream=None):
+        """Lookup and injection in one call; returns (scene, prim, weight, mask)."""
+        self._tensor(queries, "queries", self.torch_dtype)
+        hidden = list(hidden) if isinstance(hidden, (list, tuple)) else [hidden]
+        for i, h in enumerate(hidden):
+            self._tensor(h, f"hidden[{i}]", self.torch_dtype)
+        N = queries.shape[0]
+        dev = self.device
+        scene_out = torch.empty(N, dtype=torch.int32, device=dev) if scene_out is None else scene_out
+        prim_out = torch.empty(N, top_k, dtype=torch.int32, device=dev) if prim_out is None else prim_out
+        weight_out = torch.empty(N, top_k, dtype=torch.float32, device=dev) if weight_out is None else weight_out
+        mask_out = torch.empty(N, dtype=torch.uint8, device=dev) if mask_out is None else mask_out
+        arr = (ctypes.c_void_p * len(hidden))(*[h.data_ptr() for h in hidden])
+        if seg_offsets is not None:
+            seg = (ctypes.c_int64 * len(seg_offsets))(*[int(x) for x in seg_offsets])
+            n_seg = len(seg_offsets) - 1
+        else:
+            seg, n_seg = None, 0
+        _check(self.lib.lookme_lookup_inject(self.handle, _ptr(queries), N, top_k, _ptr(priority), seg, n_seg,
+                                             float(keep_ratio), arr, len(hidden), _ptr(scene_out), _ptr(prim_out),
+                                             _ptr(weight_out), _ptr(mask_out), _stream(stream, dev)))
+        return scene_out, prim_out, weight_out, mask_out
 
     def reserve(self, max_tokens):
         _check(self.lib.lookme_reserve(self.handle, max_tokens))

@@ -22,10 +22,11 @@ def _bias(w, scale, seed=11):
 
 
 def run_case(o, lookme_lib, w, *, sample=None, give_centroids=True, bias_scale=0.0, n_layers=None,
-             residency=None, table=0, mu=None, report=None, with_sel=False):
+             residency=None, table=0, mu=None, report=None, with_sel=False, fused=False):
     """with_sel requests the kept-id list, which routes the injection through
     the separate selection kernel; without it short segments take the fused
-    select + inject kernel."""
+    select + inject kernel.  fused uses lookme_lookup_inject instead of the
+    two calls."""
     from paper_2607_16305_gb300 import lookme
 
     L = n_layers or w.layers_per_table
@@ -38,12 +39,18 @@ def run_case(o, lookme_lib, w, *, sample=None, give_centroids=True, bias_scale=0
         q = W.queries(w, DEV, mu)
         hs = [W.hidden(w, l, DEV) for l in range(L)]
         h0 = [h.clone() for h in hs]
-        qn = torch.empty(N, dtype=torch.float32, device=DEV)
-        scene, prim, weight = t.lookup(q, w.top_k, qnorm_out=qn)
         n_sel = sum(int(np.floor((seg_off[i + 1] - seg_off[i]) * w.keep_ratio)) for i in range(len(seg_off) - 1))
-        sel = torch.empty(max(n_sel, 1), dtype=torch.int32, device=DEV) if with_sel else None
-        mask = t.inject(scene, prim, weight, hs, w.keep_ratio,
-                        seg_offsets=seg_off if w.n_segments > 1 else None, sel_out=sel)
+        if fused:
+            qn = None
+            with_sel = False
+            scene, prim, weight, mask = t.lookup_inject(q, w.top_k, hs, w.keep_ratio,
+                                                        seg_offsets=seg_off if w.n_segments > 1 else None)
+        else:
+            qn = torch.empty(N, dtype=torch.float32, device=DEV)
+            scene, prim, weight = t.lookup(q, w.top_k, qnorm_out=qn)
+            sel = torch.empty(max(n_sel, 1), dtype=torch.int32, device=DEV) if with_sel else None
+            mask = t.inject(scene, prim, weight, hs, w.keep_ratio,
+                            seg_offsets=seg_off if w.n_segments > 1 else None, sel_out=sel)
         torch.cuda.synchronize()
         assert t.device_status() == 0, "a device-side wait timed out"
         stats = t.stats()
@@ -72,7 +79,8 @@ def run_case(o, lookme_lib, w, *, sample=None, give_centroids=True, bias_scale=0
 
     # ---- mask / selection over all N tokens (priorities are cheap)
     qn_all = o.query_norms(H.f32(q))
-    assert np.abs(qn.cpu().numpy() - qn_all).max() <= 1e-4 * max(1.0, qn_all.max())
+    if qn is not None:
+        assert np.abs(qn.cpu().numpy() - qn_all).max() <= 1e-4 * max(1.0, qn_all.max())
     gmask = mask.cpu().numpy()
     mask_ties = H.check_mask(o, qn_all, gmask, w.keep_ratio, seg_off)
     if n_sel and with_sel:
@@ -106,9 +114,10 @@ def test_tiny_fp32_full(oracle, lookme_lib):
     run_case(oracle, lookme_lib, W.WORKLOADS["tiny_fp32"])
 
 
-@pytest.mark.parametrize("with_sel", [False, True], ids=["fused_select", "select_list"])
-def test_single_image_full(oracle, lookme_lib, with_sel):
-    res = run_case(oracle, lookme_lib, W.WORKLOADS["single_image"], with_sel=with_sel)
+@pytest.mark.parametrize("mode", ["fused_select", "select_list", "lookup_inject"])
+def test_single_image_full(oracle, lookme_lib, mode):
+    res = run_case(oracle, lookme_lib, W.WORKLOADS["single_image"], with_sel=mode == "select_list",
+                   fused=mode == "lookup_inject")
     assert res["scene_ties"] == 0
 
 
@@ -118,6 +127,7 @@ def test_batched_zipf_sampled(oracle, lookme_lib):
     rng = np.random.default_rng(0)
     run_case(oracle, lookme_lib, w, sample=rng.choice(w.n_tokens, 512, replace=False))
     run_case(oracle, lookme_lib, w, sample=rng.choice(w.n_tokens, 256, replace=False), with_sel=True)
+    run_case(oracle, lookme_lib, w, sample=rng.choice(w.n_tokens, 256, replace=False), fused=True)
 
 
 @pytest.mark.slow
@@ -125,6 +135,7 @@ def test_large_table_sampled(oracle, lookme_lib):
     w = W.WORKLOADS["large_table"]
     rng = np.random.default_rng(1)
     run_case(oracle, lookme_lib, w, sample=rng.choice(w.n_tokens, 192, replace=False))
+    run_case(oracle, lookme_lib, w, sample=rng.choice(w.n_tokens, 128, replace=False), fused=True)
 
 
 @pytest.mark.slow
@@ -134,7 +145,8 @@ def test_multilayer_host_staged_sampled(oracle, lookme_lib):
     mu = W.means(w, DEV)
     rng = np.random.default_rng(2)
     for table in (0, 6):
-        run_case(oracle, lookme_lib, w, sample=rng.choice(w.n_tokens, 256, replace=False), table=table, mu=mu)
+        run_case(oracle, lookme_lib, w, sample=rng.choice(w.n_tokens, 256, replace=False), table=table, mu=mu,
+                 fused=table == 6)
 
 
 # ---------------------------------------------------- shapes and edge cases
@@ -250,3 +262,32 @@ def test_cuda_core_variants(oracle, lookme_lib, monkeypatch, case):
     else:
         w = W.small("s6_simt", **dict(SMALL_CASES)["s6"])
     run_case(oracle, lookme_lib, w)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+@pytest.mark.parametrize("name", ["s2", "s3", "s6", "s8", "layers"])
+def test_lookup_inject_matches_separate_calls(lookme_lib, dtype, name):
+    """lookme_lookup_inject gives bit-identical results to lookme_lookup +
+    lookme_inject on the same inputs."""
+    from paper_2607_16305_gb300 import lookme
+
+    kw = dict(SMALL_CASES).get(name) or dict(n_tokens=256, n_scenes=16, n_prims=32, d_key=64, d_value=128, top_k=4,
+                                           keep_ratio=0.5)
+    w = W.small(f"li_{name}_{dtype}", dtype=dtype, **kw)
+    L = 3 if name == "layers" else 1
+    seg = w.segment_offsets if w.n_segments > 1 else None
+    with lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=w.dtype, device=0) as t:
+        H.load_table(t, w, 0, DEV)
+        q = W.queries(w, DEV)
+        h_a = [W.hidden(w, l, DEV) for l in range(L)]
+        h_b = [h.clone() for h in h_a]
+        s1, p1, w1 = t.lookup(q, w.top_k)
+        m1 = t.inject(s1, p1, w1, h_a, w.keep_ratio, seg_offsets=seg)
+        s2, p2, w2, m2 = t.lookup_inject(q, w.top_k, h_b, w.keep_ratio, seg_offsets=seg)
+        torch.cuda.synchronize()
+        assert t.device_status() == 0
+    assert torch.equal(s1, s2) and torch.equal(p1, p2) and torch.equal(w1, w2)
+    assert torch.equal(m1, m2)
+    for a, b in zip(h_a, h_b):
+        assert torch.equal(a, b)
+
