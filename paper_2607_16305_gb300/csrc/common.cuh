@@ -26,6 +26,7 @@ enum KernelId : int32_t {
     KID_CNORM = 9,       // load-time: 1 / ||centroid||
     KID_ROUTE_DECODE = 10,  // argmax key -> scene id (allocation-free routing)
     KID_SELECT_INJECT = 11, // K5 + K4 fused for short segments
+    KID_TILE_KEYS = 12,  // load-time: keys into the tcgen05 level-2 tile layout
     KID_COUNT
 };
 
@@ -165,10 +166,18 @@ struct ScoreArgs {
 cudaError_t launch_score(const LaunchCtx& c, const ScoreArgs& a);
 // Whether the level-2 kernel's shared-memory plan fits this table shape.
 bool score_shape_supported(int dtype, int64_t P, int dk);
-// Level 2 on tcgen05 (bf16 tables): tmap_keys is the CUtensorMap of the key
-// rows ([rows][d_k], box 64 x 128, 128-byte swizzle).
-cudaError_t launch_score_tc(const LaunchCtx& c, const void* tmap_keys, const ScoreArgs& a);
+// Level 2 on tcgen05 (bf16 tables).  keys_tiled holds every scene's (or
+// staging slot's) keys in the tiled layout of k_tile_keys, one block of
+// score_tc_block_bytes(P, d_k) bytes per scene; ScoreArgs::keys is unused.
+cudaError_t launch_score_tc(const LaunchCtx& c, const void* keys_tiled, const ScoreArgs& a);
 bool score_tc_shape_supported(int64_t P, int dk);
+int64_t score_tc_block_bytes(int64_t P, int dk);
+// Load time: rewrites n scenes of row-major keys [n][P][d_k] (bf16, device
+// readable) into the tiled layout: per scene, sub-blocks (tile t of 128 rows,
+// k-block b of 64 columns) in order b-major then t, each 128 rows x 128 bytes
+// with 16-byte chunk c of row r stored at chunk position c ^ (r & 7); rows
+// past P and columns past d_k are zero.
+cudaError_t launch_tile_keys(const LaunchCtx& c, const void* src, void* dst, int64_t n, int64_t P, int dk);
 // K5
 cudaError_t launch_select(const LaunchCtx& c, const float* priority, int64_t N, const int64_t* seg_off_host,
                           int n_seg, double keep_ratio, uint8_t* mask, int32_t* sel);

@@ -162,7 +162,22 @@ constexpr int kThreads = 192;
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 
 __host__ __device__ constexpr int smem_bytes(int BN, int STAGES, int nkb) {
-    return 1024 /*alignment slack*/ + nkb * BM * 128 + STAGES * BN * 128 + 256 /*barriers*/;
+    return 1024 /*alignment slack*/ + nkb * BM * 128 + STAGES * BN * 128 + 256 /*barriers*/ +
+           4 * BN * 4 /*per-tile scene constants, double-buffered*/;
+}
+
+// Named barrier 1 over the four epilogue warps, returning the OR of `v`.
+__device__ __forceinline__ bool epi_sync_or(bool v) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.or.pred q, 1, 128, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"((uint32_t)v)
+        : "memory");
+    return r != 0;
 }
 }  // namespace k1tc
 
@@ -186,6 +201,9 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
     uint64_t* drain = t_empty + 2;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
     volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    // inv ||c_s|| and bias of the current and next scene tile: [2][BN] each.
+    float* s_ic = reinterpret_cast<float*>(smem + nkb * BM * 128 + STAGES * BN * 128 + 256);
+    float* s_bias = s_ic + 2 * BN;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int m_tile = blockIdx.x;
@@ -313,50 +331,63 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
             }
             if (bias) inv_q = n > 0.f ? 1.f / n : 0.f;
         }
+        // Scene constants of the next tile are loaded while this one is scored.
+        const int et = threadIdx.x - 64;  // 0..127
+        constexpr int PER = (BN + 127) / 128;
+        float ic_next[PER], b_next[PER];
+        auto load_consts = [&](int nt) {
+#pragma unroll
+            for (int u = 0; u < PER; ++u) {
+                const int64_t s = (int64_t)nt * BN + et + u * 128;
+                const bool in = et + u * 128 < BN && s < S;
+                ic_next[u] = in ? __ldg(inv_cnorm + s) : 0.f;
+                b_next[u] = (in && bias) ? __ldg(bias + s) : 0.f;
+            }
+        };
+        auto store_consts = [&](int buf) {
+#pragma unroll
+            for (int u = 0; u < PER; ++u) {
+                if (et + u * 128 < BN) {
+                    s_ic[buf * BN + et + u * 128] = ic_next[u];
+                    s_bias[buf * BN + et + u * 128] = b_next[u];
+                }
+            }
+        };
+        if (nt0 < nt1) {
+            load_consts(nt0);
+            store_consts(0);
+        }
         unsigned long long key = 0ull;
         for (int it = 0, nt = nt0; nt < nt1; ++nt, ++it) {
             const int buf = it & 1;
             const uint32_t use = (uint32_t)(it >> 1);
-            // Warp-uniform wait: tcgen05.ld below must be executed by the whole warp.
+            if (nt + 1 < nt1) load_consts(nt + 1);
+            // Warp-uniform wait (tcgen05.ld below must be executed by the whole
+            // warp); the barrier also publishes this tile's constants.
             const bool ready = ptx::mbar_wait(&t_full[buf], use & 1u, abort, kTimeoutNs);
-            if (!__all_sync(0xFFFFFFFFu, ready)) break;
+            if (k1tc::epi_sync_or(!__all_sync(0xFFFFFFFFu, ready))) break;
             ptx::tc_fence_after();
             const int64_t s_base = (int64_t)nt * BN;
+            const float* ic = s_ic + buf * BN;
+            const float* bs = s_bias + buf * BN;
 #pragma unroll 1
             for (int c = 0; c < BN; c += 32) {
                 uint32_t r[32];
                 ptx::tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN + c), r);
                 ptx::tmem_wait_ld();
-                const int64_t s0 = s_base + c;
-                if (s0 + 32 <= S) {
-                    const float4* ic = reinterpret_cast<const float4*>(inv_cnorm + s0);
 #pragma unroll
-                    for (int j4 = 0; j4 < 8; ++j4) {
-                        const float4 w = __ldg(ic + j4);
-                        const float wv[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            const int j = j4 * 4 + u;
-                            const unsigned long long k = pack_argmax(
-                                level1_score(__uint_as_float(r[j]), wv[u], bias, s0 + j, inv_q), (uint32_t)(s0 + j));
-                            key = k > key ? k : key;
-                        }
-                    }
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        if (s0 + j < S) {
-                            const unsigned long long k =
-                                pack_argmax(level1_score(__uint_as_float(r[j]), inv_cnorm[s0 + j], bias, s0 + j, inv_q),
-                                            (uint32_t)(s0 + j));
-                            key = k > key ? k : key;
-                        }
-                    }
+                for (int j = 0; j < 32; ++j) {
+                    const int64_t s = s_base + c + j;
+                    float score = __uint_as_float(r[j]) * ic[c + j];
+                    if (bias) score = fmaf(score, inv_q, bs[c + j]);
+                    const unsigned long long k = pack_argmax(score, (uint32_t)s);
+                    if (s < S) key = k > key ? k : key;
                 }
             }
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&t_empty[buf]);
+            if (nt + 1 < nt1) store_consts(buf ^ 1);
         }
         if (row < N && key && !*abort) atomicMax(&best[row], key);
     }

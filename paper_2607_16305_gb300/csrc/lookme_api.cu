@@ -39,7 +39,8 @@ lookme_status fail(lookme_status st, const char* fmt, ...) {
 
 const char* kKernelNames[KID_COUNT] = {"prep",         "route_tc", "route_simt",    "bucket",
                                        "score",        "select",   "inject",        "stage",
-                                       "centroid_mean", "inv_cnorm", "route_decode", "select_inject"};
+                                       "centroid_mean", "inv_cnorm", "route_decode", "select_inject",
+                                       "tile_keys"};
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point, so the
 // library does not link libcuda directly.
@@ -101,7 +102,7 @@ struct lookme_table {
     int num_sms = 0;
     bool tc_route = false;  // level 1 on tcgen05
     bool tc_score = false;  // level 2 on tcgen05
-    CUtensorMap tmap_keys;  // key rows (table or slot cache) for the tcgen05 level-2 kernel
+    int64_t kblock = 0;     // bytes of one scene's stored key block (tiled when tc_score)
 
     // storage
     void* keys = nullptr;       // device, or device-mapped pinned host
@@ -345,7 +346,9 @@ lookme_status lookme_table_create(const lookme_table_desc* desc, lookme_table** 
     }
 
     const size_t S = d.n_scenes, P = d.n_prims;
-    const size_t kbytes = S * P * d.d_key * t->esz, vbytes = S * P * d.d_value * t->esz;
+    // tcgen05 tables store keys as the level-2 kernel's shared-memory tiles.
+    t->kblock = t->tc_score ? score_tc_block_bytes(d.n_prims, (int)d.d_key) : (int64_t)(P * d.d_key * t->esz);
+    const size_t kbytes = S * (size_t)t->kblock, vbytes = S * P * d.d_value * t->esz;
     bool ok = true;
     if (d.residency == LOOKME_RES_DEVICE) {
         ok = cudaMalloc(&t->keys, kbytes) == cudaSuccess && cudaMalloc(&t->values, vbytes) == cudaSuccess;
@@ -355,7 +358,7 @@ lookme_status lookme_table_create(const lookme_table_desc* desc, lookme_table** 
              cudaHostGetDevicePointer(&t->keys, t->keys_host, 0) == cudaSuccess &&
              cudaHostGetDevicePointer(&t->values, t->values_host, 0) == cudaSuccess;
         t->n_slots = d.stage_slots > 0 ? d.stage_slots : d.n_scenes;
-        ok = ok && cudaMalloc(&t->slots, (size_t)t->n_slots * P * d.d_key * t->esz) == cudaSuccess;
+        ok = ok && cudaMalloc(&t->slots, (size_t)t->n_slots * t->kblock) == cudaSuccess;
     }
     ok = ok && cudaMalloc(&t->cent, align_up(S * d.d_key * t->esz, 256)) == cudaSuccess &&
          cudaMalloc(&t->inv_cnorm, align_up(S * sizeof(float), 256)) == cudaSuccess &&
@@ -371,14 +374,6 @@ lookme_status lookme_table_create(const lookme_table_desc* desc, lookme_table** 
         cudaMemset(t->status, 0, 256) != cudaSuccess) {
         destroy_table(t);
         return fail(LOOKME_ERR_CUDA, "table initialisation failed");
-    }
-    if (t->tc_score) {
-        const bool staged = d.residency == LOOKME_RES_HOST_STAGED;
-        const int64_t rows = (staged ? t->n_slots : d.n_scenes) * d.n_prims;
-        if (!encode_bf16_2d(&t->tmap_keys, staged ? t->slots : t->keys, rows, d.d_key, 128)) {
-            destroy_table(t);
-            return fail(LOOKME_ERR_CUDA, "cuTensorMapEncodeTiled failed for the keys");
-        }
     }
     if (t->tc_route) {
         for (int i = 0; i < 3; ++i) {
@@ -439,8 +434,25 @@ lookme_status lookme_load_scenes(lookme_table* t, int64_t scene_begin, int64_t n
     char* kdst = static_cast<char*>(d.residency == LOOKME_RES_DEVICE ? t->keys : t->keys_host);
     char* vdst = static_cast<char*>(d.residency == LOOKME_RES_DEVICE ? t->values : t->values_host);
     cudaError_t e;
-    if ((e = cudaMemcpyAsync(kdst + scene_begin * krow, keys, n * krow, cudaMemcpyDefault, s)) != cudaSuccess)
-        return cuda_fail(t, e, "copy keys");
+    // Row-major keys readable by the device: the stored copy itself, or (tiled
+    // tables) a stream-ordered temporary that the tiling kernel reads.
+    const char* krows = nullptr;
+    void* ktmp = nullptr;
+    if (t->tc_score) {
+        if ((e = cudaMallocAsync(&ktmp, n * krow, s)) != cudaSuccess) return cuda_fail(t, e, "key staging buffer");
+        if ((e = cudaMemcpyAsync(ktmp, keys, n * krow, cudaMemcpyDefault, s)) != cudaSuccess)
+            return cuda_fail(t, e, "copy keys");
+        krows = static_cast<const char*>(ktmp);
+        // The tiled block goes through the device view of the destination.
+        char* tdst = static_cast<char*>(t->keys) + scene_begin * t->kblock;
+        st = launch(t, s, KID_TILE_KEYS,
+                    [&] { return launch_tile_keys(ctx, ktmp, tdst, n, d.n_prims, (int)d.d_key); });
+        if (st != LOOKME_OK) return st;
+    } else {
+        if ((e = cudaMemcpyAsync(kdst + scene_begin * krow, keys, n * krow, cudaMemcpyDefault, s)) != cudaSuccess)
+            return cuda_fail(t, e, "copy keys");
+        krows = static_cast<const char*>(t->keys) + scene_begin * krow;  // device view of the stored keys
+    }
     if ((e = cudaMemcpyAsync(vdst + scene_begin * vrow, values, n * vrow, cudaMemcpyDefault, s)) != cudaSuccess)
         return cuda_fail(t, e, "copy values");
     char* cdst = static_cast<char*>(t->cent) + scene_begin * d.d_key * t->esz;
@@ -448,11 +460,11 @@ lookme_status lookme_load_scenes(lookme_table* t, int64_t scene_begin, int64_t n
         if ((e = cudaMemcpyAsync(cdst, centroids, n * d.d_key * t->esz, cudaMemcpyDefault, s)) != cudaSuccess)
             return cuda_fail(t, e, "copy centroids");
     } else {
-        const char* ksrc = static_cast<const char*>(t->keys) + scene_begin * krow;  // device view of the stored keys
         st = launch(t, s, KID_CENTROID,
-                    [&] { return launch_centroid_mean(ctx, d.dtype, ksrc, n, d.n_prims, (int)d.d_key, cdst); });
+                    [&] { return launch_centroid_mean(ctx, d.dtype, krows, n, d.n_prims, (int)d.d_key, cdst); });
         if (st != LOOKME_OK) return st;
     }
+    if (ktmp && (e = cudaFreeAsync(ktmp, s)) != cudaSuccess) return cuda_fail(t, e, "free key staging buffer");
     st = launch(t, s, KID_CNORM, [&] {
         return launch_inv_cnorm(ctx, d.dtype, cdst, n, (int)d.d_key, t->inv_cnorm + scene_begin);
     });
@@ -524,9 +536,8 @@ lookme_status lookme_lookup(lookme_table* t, const void* queries, int64_t N, int
     if (st != LOOKME_OK) return st;
     const bool staged = d.residency == LOOKME_RES_HOST_STAGED;
     if (staged) {
-        const int64_t block_bytes = d.n_prims * d.d_key * (int64_t)t->esz;
         st = launch(t, s, KID_STAGE, [&] {
-            return launch_stage(ctx, t->keys, t->slots, block_bytes, t->n_slots, t->routed, t->counters);
+            return launch_stage(ctx, t->keys, t->slots, t->kblock, t->n_slots, t->routed, t->counters);
         });
         if (st != LOOKME_OK) return st;
     }
@@ -545,7 +556,8 @@ lookme_status lookme_lookup(lookme_table* t, const void* queries, int64_t N, int
     a.prim_out = prim_out;
     a.weight_out = weight_out;
     a.status = t->status;
-    st = launch(t, s, KID_SCORE, [&] { return t->tc_score ? launch_score_tc(ctx, &t->tmap_keys, a) : launch_score(ctx, a); });
+    st = launch(t, s, KID_SCORE,
+                [&] { return t->tc_score ? launch_score_tc(ctx, a.keys, a) : launch_score(ctx, a); });
     if (st != LOOKME_OK) return st;
     t->last_tokens = N;
     return LOOKME_OK;

@@ -14,7 +14,8 @@ __device__ __forceinline__ float from_orderable(uint32_t u) {
 }
 
 // Top-k of z[0..P) by one warp (larger z first, lower index on ties) and the
-// softmax over the selected logits; writes prim/weight of token t.
+// softmax over the selected logits; writes prim/weight of token t (nothing
+// when prim_out is null).
 __device__ __forceinline__ void topk_token(const float* z, int64_t P, int top_k, int lane, int64_t t,
                                            int32_t* prim_out, float* weight_out) {
     // Each lane keeps the best untaken element of its slice p = lane + 32 i.
@@ -67,7 +68,7 @@ __device__ __forceinline__ void topk_token(const float* z, int64_t P, int top_k,
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
         const int j = h * 32 + lane;
-        if (j < top_k) {
+        if (j < top_k && prim_out) {
             prim_out[t * top_k + j] = my_p[h];
             weight_out[t * top_k + j] = e[h] / sum;
         }
@@ -126,7 +127,7 @@ __device__ __forceinline__ void topk_token_regs(const float* z, int64_t P, int t
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
         const int j = h * 32 + lane;
-        if (j < top_k) {
+        if (j < top_k && prim_out) {
             prim_out[t * top_k + j] = my_p[h];
             weight_out[t * top_k + j] = e[h] / sum;
         }
