@@ -174,9 +174,9 @@ bool score_tc_shape_supported(int64_t P, int dk);
 int64_t score_tc_block_bytes(int64_t P, int dk);
 // Load time: rewrites n scenes of row-major keys [n][P][d_k] (bf16, device
 // readable) into the tiled layout: per scene, sub-blocks (tile t of 128 rows,
-// k-block b of 64 columns) in order b-major then t, each 128 rows x 128 bytes
-// with 16-byte chunk c of row r stored at chunk position c ^ (r & 7); rows
-// past P and columns past d_k are zero.
+// k-block b of 64 columns) ordered by N-tile (tiles 2m, 2m + 1), then b, then
+// t, each 128 rows x 128 bytes with 16-byte chunk c of row r stored at chunk
+// position c ^ (r & 7); rows past P and columns past d_k are zero.
 cudaError_t launch_tile_keys(const LaunchCtx& c, const void* src, void* dst, int64_t n, int64_t P, int dk);
 // K5
 cudaError_t launch_select(const LaunchCtx& c, const float* priority, int64_t N, const int64_t* seg_off_host,

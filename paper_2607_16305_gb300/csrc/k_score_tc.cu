@@ -3,39 +3,46 @@
 //   z_tp = q_t . K[j, p] / sqrt(d_k), I_t = top-k of z_t, w_t = softmax(z_t[I_t]).
 //
 // Each work item (a scene and <= 8 of its tokens) is a small grouped GEMM:
-// D[p][j] = K[scene, p, :] . q_j for the scene's N_p key rows and the item's
-// tokens.  The keys are the M = 128 operand, the tokens the N = 16 operand (a
-// swizzled K-major tile built in shared memory from bulk-copied query rows),
-// and the fp32 accumulator lives in TMEM.
+// D[j][p] = q_j . K[scene, p, :] for the item's tokens and the scene's N_p
+// key rows.  The keys are the N operand, up to 256 rows per MMA (an "N-tile"),
+// because a tcgen05.mma costs about the same time whatever its N: with the
+// keys as N = 256 each MMA consumes 8 KiB of keys, twice what the 128-row M
+// operand would.  The tokens are the M = 128 operand: one 1 KiB swizzled
+// atom of 8 token rows per 64-wide k-block, with the descriptor's atom stride
+// set to zero so that every 8-row group of M reads the same atom (D row r is
+// token r % 8).  The fp32 accumulator D lives in TMEM, two buffers of 256
+// columns.
 //
 // The table stores every scene's keys as the exact shared-memory image the
-// MMA reads: sub-blocks of 128 rows x 64 columns (16 KiB, 128-byte swizzle),
-// k-block-major then row tile, zero-padded past N_p and d_k.  A scene's block is
-// therefore contiguous and is streamed with 1-D bulk copies of up to four
-// sub-blocks (64 KiB): a copy costs the SM's copy engine about the same time
-// whatever its size in this range, so large copies are what lets one CTA per
-// SM pull its share of HBM bandwidth.
+// MMA reads: 128-row x 64-column sub-blocks (16 KiB, 128-byte swizzle),
+// ordered N-tile, then k-block, then the N-tile's one or two sub-blocks
+// (which are adjacent, so an N = 256 operand is one contiguous 32 KiB), and
+// zero-padded past N_p and d_k.  A scene's block is contiguous and is
+// streamed with 1-D bulk copies of up to four sub-blocks: the copy engine of
+// an SM spends about the same time on a 16 KiB and a 64 KiB copy, so large
+// copies are what lets one CTA per SM pull its share of HBM bandwidth.
 //
-// With N = 16 each MMA is short, and back-to-back MMAs into one accumulator
-// wait on each other; so each row tile accumulates into nacc partial sums
-// (k-block b goes to partial b % nacc) and a copy's MMAs are issued k-step by
-// k-step across its sub-blocks, which keeps several independent
-// accumulations in flight.  The epilogue adds the partials.  The tensor core
-// removes the CUDA-core work that would otherwise have to keep pace with the
-// key stream.  One CTA
-// per SM, static share of the work list (items b, b + G, b + 2G, ...):
+// One CTA per SM, static share of the work list (items b, b + G, ...):
 //   warp 0       producer: reads each item's work entry and streams the
 //                scene's key block through the ring (bulk copies only)
-//   warp 1       one thread issues tcgen05.mma into one of two TMEM buffers
-//   warps 2..9   epilogue: TMEM -> logits in shared memory (scaled), then
-//                top-k + softmax, one token per warp (redux.sync argmax)
-//   warp 10      token tiles: reads the item's token ids and query rows with
+//   warp 1       one thread issues tcgen05.mma, N-tile by N-tile, into the
+//                two TMEM buffers
+//   warps 2..17  epilogue, two groups of eight taking alternate items (so one
+//                item's top-k overlaps the next item's read-out): TMEM ->
+//                logits in shared memory (scaled), then top-k + softmax, one
+//                token per warp
+//   warp 18      token tiles: reads the item's token ids and query rows with
 //                plain 16-byte loads and writes them straight into the
-//                swizzled K-major tile (small copies would each cost the
-//                copy engine as much time as a 64 KiB one)
+//                swizzled tile (small copies would each cost the copy engine
+//                as much time as a 64 KiB one)
+// Before the grid dependency wait, the MMA issuer and the top-k run once
+// without effect, so their code is cached before the key stream starts (a
+// first instruction fetch under the full stream costs microseconds).
 // Every wait is bounded; on a timeout the kernel drains its copies and MMAs,
 // releases TMEM and reports through the status word.
 #include <cuda.h>
+
+#include <algorithm>
 
 #include "common.cuh"
 #include "sm100.cuh"
@@ -44,18 +51,19 @@
 namespace lookme {
 
 namespace k3tc {
-constexpr int BM = 128;                  // key rows per MMA tile
 constexpr int BK = 64;                   // bf16 elements per 128-byte swizzled row
-constexpr int BN = 16;                   // token columns (an item holds <= 8 tokens)
-constexpr int kTok = kTokensPerItem;
-constexpr int kSubBytes = BM * 128;      // one 128 x 64 key sub-block: 16 KiB
-constexpr int kBKbBytes = BN * 128;      // one 16 x 64 token block: 2 KiB
-constexpr int kEpiWarps = 8;
+constexpr int kSubRows = 128;            // key rows per sub-block
+constexpr int kNTile = 256;              // key rows per MMA (N)
+constexpr int kTok = kTokensPerItem;     // token rows of the A atom
+constexpr int kSubBytes = kSubRows * 128;  // one 128 x 64 key sub-block: 16 KiB
+constexpr int kAtomBytes = 1024;         // 8 token rows x 128 bytes per k-block
+constexpr int kZStride = 9;              // logits z[p][j] at p * 9 + j: conflict-free both ways
+constexpr int kGroupWarps = 8;           // epilogue warps per item group (one token each)
+constexpr int kEpiWarps = 2 * kGroupWarps;
 constexpr int kBuildWarp = 2 + kEpiWarps;
 constexpr int kThreads = (3 + kEpiWarps) * 32;
-constexpr int kQBatch = 8;               // query-row chunks in flight per lane
-constexpr int kMaxStages = 14;          // ring slots (barrier arrays)
-constexpr int kMaxGroup = 4;             // sub-blocks per bulk copy / ring slot
+constexpr int kQBatch = 4;               // query-row chunks in flight per lane
+constexpr int kMaxStages = 14;           // ring slots (barrier arrays)
 constexpr int kBSlots = 2;               // token tiles
 constexpr int kISlots = 4;               // item metadata (scene, count, token ids)
 constexpr uint64_t kTimeoutNs = 1000000000ull;
@@ -63,16 +71,18 @@ constexpr int kSmemLimit = 227 * 1024;
 
 struct Geometry {
     int nkb;              // 64-wide k-blocks of d_k
-    int ntile;            // 128-row tiles of N_p
-    int group;            // sub-blocks per ring slot (one bulk copy)
+    int ntile;            // 128-row sub-block rows of N_p
+    int nnt;              // N-tiles (256 rows; the last may hold one sub-block)
+    int spi;              // sub-blocks per item (ntile x nkb)
+    int group;            // sub-blocks per ring slot (one bulk copy): 4, 2 or 1
+    int gshift;           // log2(group)
     int slot_bytes;       // group x 16 KiB
     int n_stages;         // ring slots
-    int spi;              // sub-blocks per item (ntile x nkb)
     int chunks;           // bulk copies per item
     int row_bytes;        // d_k * 2
-    int b_bytes;          // one token tile (nkb x 2 KiB)
-    int nacc;             // partial accumulators per row tile
-    int tmem_cols;        // allocated TMEM columns (two buffers of ntile x nacc x 16)
+    int b_bytes;          // one token tile (nkb x 1 KiB)
+    int tmem_cols;        // two D buffers
+    int zbytes;           // logits of one item (per epilogue group)
     int off_b, off_z, off_bar, off_meta;
     int smem;             // bytes requested, including 1 KiB of alignment slack
 };
@@ -80,91 +90,90 @@ struct Geometry {
 inline Geometry geometry(int64_t P, int dk) {
     Geometry g;
     g.nkb = (dk + BK - 1) / BK;
-    g.ntile = (int)((P + BM - 1) / BM);
-    g.row_bytes = dk * 2;
-    g.b_bytes = g.nkb * kBKbBytes;
-    g.nacc = min(4, g.nkb);
-    while (g.nacc > 1 && 2 * g.ntile * g.nacc * BN > 512) --g.nacc;
-    int cols = 32;
-    while (cols < 2 * g.ntile * g.nacc * BN) cols <<= 1;
-    g.tmem_cols = cols;
-    const int zbytes = (kTok * (int)P * 4 + 15) / 16 * 16;
-    const int fixed = kBSlots * g.b_bytes + zbytes + 1024 /*bar+meta*/ + 1024 /*align*/;
+    g.ntile = (int)((P + kSubRows - 1) / kSubRows);
+    g.nnt = (g.ntile + 1) / 2;
     g.spi = g.ntile * g.nkb;
-    // The largest copies that still leave at least two ring slots.
-    g.group = kMaxGroup;
-    while (g.group > 1 && (kSmemLimit - fixed) / (g.group * kSubBytes) < 2) g.group >>= 1;
-    if (g.group > g.spi) g.group = g.spi;
+    g.row_bytes = dk * 2;
+    g.b_bytes = g.nkb * kAtomBytes;
+    const int nmax = (int)std::min<int64_t>(kNTile, (P + 15) / 16 * 16);
+    int cols = 32;
+    while (cols < 2 * nmax) cols <<= 1;
+    g.tmem_cols = cols;
+    g.zbytes = ((int)P * kZStride * 4 + 15) / 16 * 16;  // per epilogue group
+    const int fixed = kBSlots * g.b_bytes + 2 * g.zbytes + 1024 /*bar+meta*/ + 1024 /*align*/;
+    // The largest copies that leave at least two ring slots; a two-sub-block
+    // N-tile unit must fit in one slot, and units start at even sub-blocks.
+    g.gshift = 2;
+    while (g.gshift > 0 && (kSmemLimit - fixed) / ((kSubBytes << g.gshift)) < 2) --g.gshift;
+    while (g.gshift > 0 && (1 << g.gshift) > g.spi) --g.gshift;
+    g.group = 1 << g.gshift;
     g.slot_bytes = g.group * kSubBytes;
     g.chunks = (g.spi + g.group - 1) / g.group;
     g.n_stages = (kSmemLimit - fixed) / g.slot_bytes;
     if (g.n_stages > kMaxStages) g.n_stages = kMaxStages;
     g.off_b = g.n_stages * g.slot_bytes;
     g.off_z = g.off_b + kBSlots * g.b_bytes;
-    g.off_bar = g.off_z + zbytes;
+    g.off_bar = g.off_z + 2 * g.zbytes;
     g.off_meta = g.off_bar + (2 * kMaxStages + 2 * kBSlots + 2 * kISlots + 2 * 2 + 1) * 8;
     g.smem = g.off_meta + kISlots * ((int)sizeof(WorkItem) + kTok * 4) + 16 + 1024;
     return g;
 }
 
-// Named barrier 1 over the epilogue warps, returning the OR of `v` over them.
-__device__ __forceinline__ bool epi_sync_or(bool v) {
+// Named barrier 1 + grp over one epilogue group, returning the OR of `v` over it.
+template <int ID>
+__device__ __forceinline__ bool bar_or(bool v) {
     uint32_t r;
     asm volatile(
         "{\n\t.reg .pred p, q;\n\t"
         "setp.ne.u32 p, %1, 0;\n\t"
-        "bar.red.or.pred q, 1, %2, p;\n\t"
+        "bar.red.or.pred q, %2, %3, p;\n\t"
         "selp.u32 %0, 1, 0, q;\n\t}"
         : "=r"(r)
-        : "r"((uint32_t)v), "n"(kEpiWarps * 32)
+        : "r"((uint32_t)v), "n"(ID), "n"(kGroupWarps * 32)
         : "memory");
     return r != 0;
 }
-// Position in an item's sub-blocks (k-block-major, then row tile).
-struct SubCursor {
-    int kb, tile, kbm;  // k-block, row tile, kb % nacc
-};
+__device__ __forceinline__ bool group_sync_or(int grp, bool v) { return grp == 0 ? bar_or<1>(v) : bar_or<2>(v); }
 
-// Issues the MMAs of one ring slot's nsub sub-blocks, k-step by k-step across
-// the sub-blocks so that consecutive MMAs go to different accumulators, and
-// returns the cursor past them.  live = 0 runs the same instructions with
-// every MMA switched off: called once before the grid dependency wait, it
-// pulls this code into the instruction cache while memory is quiet (a first
-// fetch under the full key stream costs several microseconds).  One copy of
-// the code serves both calls.
-__device__ __noinline__ SubCursor mma_chunk(uint32_t live, SubCursor cur, int nsub, uint32_t dbase, uint64_t ad,
-                                            uint64_t bd, int ntile, int nacc) {
-    constexpr uint32_t idesc = ptx::idesc_bf16_f32<BM, BN>();
-    constexpr uint32_t kSubUnits = kSubBytes >> 4, kKbUnits = kBKbBytes >> 4, kKUnits = 32 >> 4;
-    uint32_t dcol[kMaxGroup], boff[kMaxGroup], acc0[kMaxGroup];
-#pragma unroll
-    for (int j = 0; j < kMaxGroup; ++j) {
-        dcol[j] = dbase + (uint32_t)((cur.tile * nacc + cur.kbm) * BN);
-        boff[j] = (uint32_t)cur.kb * kKbUnits;
-        acc0[j] = cur.kb >= nacc ? 1u : 0u;  // a partial's first k-block overwrites at its first k-step
-        if (j < nsub && ++cur.tile == ntile) {
-            cur.tile = 0;
-            ++cur.kb;
-            if (++cur.kbm == nacc) cur.kbm = 0;
-        }
-    }
-#pragma unroll
-    for (int k = 0; k < BK / 16; ++k) {
-#pragma unroll
-        for (int j = 0; j < kMaxGroup; ++j) {
-            if (j < nsub)
-                ptx::mma_bf16_if(live, dcol[j], ad + (uint64_t)(j * kSubUnits + k * kKUnits),
-                                 bd + (uint64_t)(boff[j] + k * kKUnits), idesc, k != 0 ? 1u : acc0[j]);
-        }
-    }
-    return cur;
+// Shared-memory descriptor of a K-major, 128-byte-swizzled operand whose
+// 8-row atoms are `sbo` bytes apart (0: every atom is the same 1 KiB).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr, uint32_t sbo) {
+    return (ptx::sw128_kmajor_desc(saddr) & ~(0x3FFFull << 32)) | ((uint64_t)(sbo >> 4) << 32);
 }
 
-// Top-k + softmax of one token; a single copy serves the warm-up call
-// (prim_out == nullptr: nothing is written) and the real ones.
-__device__ __noinline__ void topk_item(const float* z, int64_t P, int top_k, int lane, int64_t t, int32_t* prim_out,
-                                       float* weight_out) {
-    k3::topk_any(z, P, top_k, lane, t, prim_out, weight_out);
+// Instruction descriptor of kind::f16, bf16 A and B, fp32 D, M = 128, N = n.
+__device__ __forceinline__ uint32_t idesc_m128(int n) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+}
+
+// The four k-steps of one 64-wide k-block of an N-tile.  live = 0 runs the
+// same instructions with every MMA switched off (the warm-up call); one copy
+// of the code serves both.
+__device__ __noinline__ void mma_kblock(uint32_t live, uint32_t d, uint64_t ad, uint64_t bd, uint32_t idesc,
+                                        uint32_t first) {
+#pragma unroll
+    for (int k = 0; k < BK / 16; ++k)
+        ptx::mma_bf16_if(live, d, ad + (uint64_t)(k * 2), bd + (uint64_t)(k * 2), idesc,
+                         (first && k == 0) ? 0u : 1u);
+}
+
+// Top-k + softmax of one token over logits at stride kZStride; a single copy
+// serves the warm-up call (prim_out == nullptr: nothing is written) and the
+// real ones.  The common shape (N_p <= 256, top_k <= 8) has a function of its
+// own, so that the larger variants' registers do not weigh on it.
+__device__ __noinline__ void topk_small(const float* z, int64_t P, int top_k, int lane, int64_t t,
+                                        int32_t* prim_out, float* weight_out) {
+    if (P <= 64) k3::topk_token_pop<2, 8>(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
+    else k3::topk_token_pop<8, 8>(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
+}
+__device__ __noinline__ void topk_large(const float* z, int64_t P, int top_k, int lane, int64_t t,
+                                        int32_t* prim_out, float* weight_out) {
+    k3::topk_any(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
+}
+__device__ __forceinline__ void topk_item(const float* z, int64_t P, int top_k, int lane, int64_t t,
+                                          int32_t* prim_out, float* weight_out) {
+    if (P <= 256 && top_k <= 8) topk_small(z, P, top_k, lane, t, prim_out, weight_out);
+    else topk_large(z, P, top_k, lane, t, prim_out, weight_out);
 }
 }  // namespace k3tc
 
@@ -196,12 +205,9 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
 
     const int tid = threadIdx.x, lane = tid % 32, warp = tid / 32;
     pdl_trigger();
-    // While the predecessor finishes, run the MMA issuer and the top-k once
-    // without effect, so their code is cached before the key stream starts.
+    // Warm-up while the predecessor finishes: no memory, barrier or TMEM effect.
     if (warp == 1 && lane == 0) {
-        SubCursor cur{0, 0, 0};
-        for (int c = 0; c < min(g.chunks, 2); ++c) cur = mma_chunk(0u, cur, min(g.group, g.spi), 0u, 0ull, 0ull,
-                                                                 g.ntile, g.nacc);
+        mma_kblock(0u, 0u, 0ull, 0ull, idesc_m128(kNTile), 1u);
     } else if (warp >= 2 && warp < kBuildWarp) {
         topk_item(zs, P, top_k, lane, 0, nullptr, nullptr);
     }
@@ -213,6 +219,13 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
     const int my_items = n_work > (int)blockIdx.x ? (n_work - (int)blockIdx.x + G - 1) / G : 0;
     if (my_items == 0) return;  // uniform for the CTA: nothing allocated yet
     auto item_index = [&](int i) { return (int)blockIdx.x + i * G; };
+    // N-tile nt: its first sub-block, its sub-block count (1 or 2) and its N.
+    auto nt_base = [&](int nt) { return nt * 2 * g.nkb; };
+    auto nt_subs = [&](int nt) { return (nt == g.nnt - 1 && (g.ntile & 1)) ? 1 : 2; };
+    auto nt_cols = [&](int nt) {
+        const int64_t rows = P - (int64_t)nt * kNTile;
+        return (int)(rows >= kNTile ? kNTile : (rows + 15) / 16 * 16);
+    };
 
     if (tid == 0) {
         for (int i = 0; i < g.n_stages; ++i) {
@@ -225,11 +238,11 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         }
         for (int i = 0; i < kISlots; ++i) {
             ptx::mbar_init(&ifull[i], 1);
-            ptx::mbar_init(&iempty[i], kEpiWarps);
+            ptx::mbar_init(&iempty[i], kGroupWarps);
         }
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(&dready[i], 1);
-            ptx::mbar_init(&tempty[i], kEpiWarps);
+            ptx::mbar_init(&tempty[i], kGroupWarps);
         }
         ptx::mbar_init(drain, 1);
         *abort = 0;
@@ -284,39 +297,54 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
     } else if (warp == 1) {
         // ------------------------------------------------------------- MMA
         if (lane == 0) {
-            // Operand descriptors advance by adding 16-byte units to their start
-            // address field (shared addresses stay below 2^18: no carry out of it).
-            const uint64_t ad_ring = ptx::sw128_kmajor_desc(ptx::smem_u32(ring));
-            const uint64_t bd_tiles = ptx::sw128_kmajor_desc(ptx::smem_u32(btile));
+            const uint32_t a_tiles = ptx::smem_u32(btile);
             int slot = 0;
             uint32_t phase = 0;
+            int qn = 0;  // N-tiles issued (D buffer qn & 1)
             bool ok = true;
             for (int i = 0; i < my_items && ok; ++i) {
-                const int bs = i % kBSlots, d = i & 1;
-                ok = ptx::mbar_wait(&bfull[bs], (i / kBSlots) & 1, abort, kTimeoutNs) &&
-                     ptx::mbar_wait(&tempty[d], ((i >> 1) & 1) ^ 1, abort, kTimeoutNs);
-                if (!ok) break;
+                const int bs = i % kBSlots;
+                if (!(ok = ptx::mbar_wait(&bfull[bs], (i / kBSlots) & 1, abort, kTimeoutNs))) break;
                 ptx::tc_fence_after();
-                const uint32_t dbase = tmem_base + (uint32_t)(d * g.ntile * g.nacc * BN);
-                const uint64_t bd = bd_tiles + (uint64_t)((bs * g.b_bytes) >> 4);
-                SubCursor cur{0, 0, 0};
-                for (int c = 0, done = 0; c < g.chunks; ++c) {
-                    if (!(ok = ptx::mbar_wait(&full[slot], phase, abort, kTimeoutNs))) break;
+                const uint64_t ad0 = sw128_desc(a_tiles + (uint32_t)(bs * g.b_bytes), 0);
+                int cur_chunk = -1;
+                for (int nt = 0; nt < g.nnt && ok; ++nt, ++qn) {
+                    const int buf = qn & 1;
+                    if (!(ok = ptx::mbar_wait(&tempty[buf], ((qn >> 1) & 1) ^ 1, abort, kTimeoutNs))) break;
                     ptx::tc_fence_after();
-                    const int nsub = min(g.group, g.spi - done);
-                    cur = mma_chunk(1u, cur, nsub, dbase, ad_ring + (uint64_t)((slot * g.slot_bytes) >> 4), bd,
-                                    g.ntile, g.nacc);
-                    ptx::mma_commit(&empty[slot]);
-                    done += nsub;
-                    if (++slot == g.n_stages) {
-                        slot = 0;
-                        phase ^= 1u;
+                    const uint32_t d = tmem_base + (uint32_t)(buf * (g.tmem_cols >> 1));
+                    const uint32_t idesc = idesc_m128(nt_cols(nt));
+                    const int ns = nt_subs(nt);
+                    for (int kb = 0; kb < g.nkb; ++kb) {
+                        const int sb = nt_base(nt) + kb * ns;
+                        const int ch = sb >> g.gshift;
+                        if (ch != cur_chunk) {
+                            if (cur_chunk >= 0) {
+                                ptx::mma_commit(&empty[slot]);
+                                if (++slot == g.n_stages) {
+                                    slot = 0;
+                                    phase ^= 1u;
+                                }
+                            }
+                            if (!(ok = ptx::mbar_wait(&full[slot], phase, abort, kTimeoutNs))) break;
+                            ptx::tc_fence_after();
+                            cur_chunk = ch;
+                        }
+                        const uint32_t b_addr = ptx::smem_u32(ring + (int64_t)slot * g.slot_bytes +
+                                                              (int64_t)(sb - (ch << g.gshift)) * kSubBytes);
+                        mma_kblock(1u, d, ad0 + (uint64_t)(kb * (kAtomBytes >> 4)), sw128_desc(b_addr, 1024), idesc,
+                                   kb == 0 ? 1u : 0u);
                     }
+                    if (ok) ptx::mma_commit(&dready[buf]);
                 }
-                if (ok) {
-                    ptx::mma_commit(&bempty[bs]);
-                    ptx::mma_commit(&dready[d]);
+                if (!ok) break;
+                // The item's last copy and its token tile are free once these MMAs complete.
+                ptx::mma_commit(&empty[slot]);
+                if (++slot == g.n_stages) {
+                    slot = 0;
+                    phase ^= 1u;
                 }
+                ptx::mma_commit(&bempty[bs]);
             }
             // All MMAs complete before TMEM is released and the CTA exits.
             ptx::mma_commit(drain);
@@ -324,44 +352,47 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         }
     } else if (warp < kBuildWarp) {
         // -------------------------------------------------------- epilogue
-        const int e = warp - 2;           // 0..7
+        const int e = warp - 2;
+        const int grp = e / kGroupWarps;  // takes items grp, grp + 2, ...
+        const int eg = e % kGroupWarps;   // token of the top-k, column slice of the read-out
         const int quarter = warp & 3;     // TMEM lanes this warp may access
-        const int half = e >> 2;          // the two warps of a quarter split the row tiles
-        for (int i = 0; i < my_items; ++i) {
-            const int ms = i % kISlots, d = i & 1;
-            bool ok = ptx::mbar_wait(&ifull[ms], (i / kISlots) & 1, abort, kTimeoutNs) &&
-                      ptx::mbar_wait(&dready[d], (i >> 1) & 1, abort, kTimeoutNs);
-            ok = __all_sync(0xFFFFFFFFu, ok);
-            // Also orders this item's logit writes after every warp's top-k of the previous item.
-            if (k3tc::epi_sync_or(!ok || *abort)) break;
+        float* zg = zs + grp * (g.zbytes / 4);
+        for (int i = grp; i < my_items; i += 2) {
+            const int ms = i % kISlots;
+            bool ok = __all_sync(0xFFFFFFFFu, ptx::mbar_wait(&ifull[ms], (i / kISlots) & 1, abort, kTimeoutNs));
+            // Also orders this item's logit writes after the group's top-k of its previous item.
+            if (k3tc::group_sync_or(grp, !ok || *abort)) break;
             const int nb = min(items[ms].count, kTok);
-            ptx::tc_fence_after();
-            for (int tile = half; tile < g.ntile; tile += 2) {
-                float acc[kTok];
+            for (int nt = 0; nt < g.nnt; ++nt) {
+                const int qn = i * g.nnt + nt, buf = qn & 1;
+                ok = __all_sync(0xFFFFFFFFu, ptx::mbar_wait(&dready[buf], (qn >> 1) & 1, abort, kTimeoutNs));
+                const int ncols = nt_cols(nt);
+                // Warp eg reads columns [32 eg, 32 eg + 32) of its lanes; lane j < 8 of any
+                // quarter holds token j (D row r is token r % 8).
+                const int c0 = eg * 32;
+                if (ok && c0 < ncols) {
+                    ptx::tc_fence_after();
+                    const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) +
+                                           (uint32_t)(buf * (g.tmem_cols >> 1) + c0);
+#pragma unroll 1
+                    for (int h = 0; h < 32 && c0 + h < ncols; h += 16) {
+                        uint32_t r[16];
+                        ptx::tmem_ld_32x32b_x16(taddr + (uint32_t)h, r);
+                        ptx::tmem_wait_ld();
+                        if (lane < nb) {
+                            const int64_t p0 = (int64_t)nt * kNTile + c0 + h;
 #pragma unroll
-                for (int j = 0; j < kTok; ++j) acc[j] = 0.f;
-                const uint32_t tbase = tmem_base + ((uint32_t)(quarter * 32) << 16) +
-                                       (uint32_t)((d * g.ntile + tile) * g.nacc * BN);
-                for (int a = 0; a < g.nacc; ++a) {
-                    uint32_t r[16];
-                    ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)(a * BN), r);
-                    ptx::tmem_wait_ld();
-#pragma unroll
-                    for (int j = 0; j < kTok; ++j) acc[j] += __uint_as_float(r[j]);
+                            for (int j = 0; j < 16; ++j)
+                                if (p0 + j < P) zg[(p0 + j) * kZStride + lane] = __uint_as_float(r[j]) * scale;
+                        }
+                    }
                 }
-                const int64_t p = (int64_t)tile * BM + quarter * 32 + lane;
-                if (p < P) {
-#pragma unroll
-                    for (int j = 0; j < kTok; ++j)
-                        if (j < nb) zs[j * P + p] = acc[j] * scale;
-                }
+                ptx::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&tempty[buf]);
             }
-            ptx::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&tempty[d]);
-            if (k3tc::epi_sync_or(*abort)) break;  // all logits of the item are in shared memory
-            for (int j = e; j < nb; j += kEpiWarps)
-                k3tc::topk_item(zs + j * P, P, top_k, lane, toks[ms * kTok + j], prim_out, weight_out);
+            if (k3tc::group_sync_or(grp, *abort)) break;  // all logits of the item are in shared memory
+            if (eg < nb) k3tc::topk_item(zg + eg, P, top_k, lane, toks[ms * kTok + eg], prim_out, weight_out);
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&iempty[ms]);
         }
@@ -403,8 +434,9 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
 #pragma unroll
                 for (int u = 0; u < kQBatch; ++u) {
                     if (cc[u] >= 0) {
+                        // Row j of k-block kb: 16-byte chunk c at position c ^ j (j < 8).
                         const int j = jj[u], kb = cc[u] >> 3, c = cc[u] & 7;
-                        *reinterpret_cast<uint4*>(bt + kb * kBKbBytes + j * 128 + ((c ^ (j & 7)) * 16)) = v[u];
+                        *reinterpret_cast<uint4*>(bt + kb * kAtomBytes + j * 128 + ((c ^ j) * 16)) = v[u];
                     }
                 }
             }
@@ -434,7 +466,8 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
 
 bool score_tc_shape_supported(int64_t P, int dk) {
     const k3tc::Geometry g = k3tc::geometry(P, dk);
-    return g.n_stages >= 2 && g.smem <= k3tc::kSmemLimit && g.tmem_cols <= 512 && (dk % 8) == 0;
+    return g.n_stages >= 2 && g.smem <= k3tc::kSmemLimit && g.tmem_cols <= 512 && (dk % 8) == 0 &&
+           (g.ntile < 2 || g.group >= 2);
 }
 
 int64_t score_tc_block_bytes(int64_t P, int dk) {

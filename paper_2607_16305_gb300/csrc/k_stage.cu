@@ -43,8 +43,11 @@ __global__ void __launch_bounds__(256) k6_stage(const uint4* __restrict__ keys_h
 }
 
 // Load time: keys of n scenes, row-major [n][P][d_k] bf16, into the tiled
-// layout the tcgen05 level-2 kernel copies straight into shared memory.  One
-// thread per 16-byte output chunk, so the writes are coalesced.
+// layout the tcgen05 level-2 kernel copies straight into shared memory: per
+// scene, for each N-tile of 256 rows (the last may be 128), for each 64-wide
+// k-block, the N-tile's 128-row sub-blocks; each sub-block is 128 rows x 128
+// bytes with 16-byte chunk c of row r at position c ^ (r & 7).  One thread per
+// 16-byte output chunk, so the writes are coalesced.
 __global__ void __launch_bounds__(256) k_tile_keys(const uint4* __restrict__ src, uint4* __restrict__ dst,
                                                    int64_t n, int64_t P, int row_chunks, int ntile, int nkb) {
     const int64_t per_scene = (int64_t)ntile * nkb * 128 * 8;
@@ -55,7 +58,11 @@ __global__ void __launch_bounds__(256) k_tile_keys(const uint4* __restrict__ src
         const int64_t rem = i - s * per_scene;
         const int sb = (int)(rem >> 10), w = (int)(rem & 1023);
         const int r = w >> 3, pos = w & 7;
-        const int kb = sb / ntile, tile = sb - kb * ntile;
+        // Sub-block sb: N-tile nt (two 128-row tiles, the last maybe one), then
+        // k-block kb, then the tile within the N-tile.
+        const int nt = sb / (2 * nkb), in_nt = sb - nt * 2 * nkb;
+        const int ns = (2 * nt + 1 < ntile) ? 2 : 1;
+        const int kb = in_nt / ns, tile = 2 * nt + (in_nt - kb * ns);
         const int64_t p = (int64_t)tile * 128 + r;
         const int kc = kb * 8 + (pos ^ (r & 7));  // 16-byte chunk of the source row
         uint4 v = make_uint4(0u, 0u, 0u, 0u);
