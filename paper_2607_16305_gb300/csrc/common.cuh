@@ -166,10 +166,29 @@ struct ScoreArgs {
 cudaError_t launch_score(const LaunchCtx& c, const ScoreArgs& a);
 // Whether the level-2 kernel's shared-memory plan fits this table shape.
 bool score_shape_supported(int dtype, int64_t P, int dk);
+// The injection gate computed inside the tcgen05 level-2 kernel (by warps
+// that would otherwise wait for the first keys): token t of segment s is kept
+// iff its rank (larger priority first, lower index on ties) is below
+// r_s = floor(len_s * keep_ratio); kept tokens go to sel[sel_base[s] + rank].
+constexpr int kMaxGateSegments = 64;
+struct GateSpec {
+    int enabled;
+    int n_seg;
+    int64_t N;
+    double keep_ratio;
+    const float* priority;
+    uint8_t* mask;
+    int32_t* sel;
+    int64_t off[kMaxGateSegments + 1];
+    int64_t sel_base[kMaxGateSegments];
+};
+
 // Level 2 on tcgen05 (bf16 tables).  keys_tiled holds every scene's (or
 // staging slot's) keys in the tiled layout of k_tile_keys, one block of
 // score_tc_block_bytes(P, d_k) bytes per scene; ScoreArgs::keys is unused.
-cudaError_t launch_score_tc(const LaunchCtx& c, const void* keys_tiled, const ScoreArgs& a);
+// gate (optional) adds the injection gate.
+cudaError_t launch_score_tc(const LaunchCtx& c, const void* keys_tiled, const ScoreArgs& a,
+                            const GateSpec* gate = nullptr);
 bool score_tc_shape_supported(int64_t P, int dk);
 int64_t score_tc_block_bytes(int64_t P, int dk);
 // Load time: rewrites n scenes of row-major keys [n][P][d_k] (bf16, device

@@ -244,88 +244,125 @@ __global__ void __launch_bounds__(k4::kThreads) k4_inject(const __grid_constant_
 }
 
 // Selection fused into the injection (segments of at most kFusedMaxSegment
-// tokens): one CTA per token computes the token's rank in its segment,
+// tokens): a CTA takes two consecutive tokens and computes each one's rank in
+// its segment,
 //   rank_t = #{ j : pi_j > pi_t, or pi_j == pi_t and j < t },
 // which orders tokens exactly like the radix selection (larger priority
-// first, lower index on ties); the token is kept iff rank_t < r.  Kept tokens
-// are injected by the same CTA.  Every load the rank and the row addresses
-// need is issued before any is used, so the kernel costs one L2 round trip
-// for the gate and one HBM round trip for the injection.
+// first, lower index on ties); a token is kept iff rank_t < r.  The same CTA
+// injects its kept tokens.  Every load the ranks and the row addresses need
+// is issued before any is used (one L2 round trip for the gate, one HBM round
+// trip per kept token), and two tokens per CTA keep the whole grid of a
+// 1,024-token call resident at once.
 namespace k45 {
 constexpr int kThreads = 256;  // one 16-byte chunk of a 2,048-wide bf16 row per thread
+constexpr int kTPC = 2;        // tokens per CTA (the code below spells out two)
 constexpr int kUnroll = 4;     // priorities in flight per thread and pass
-}  // namespace k45
+constexpr int kWarps = kThreads / 32;
 
-template <typename T>
-__global__ void __launch_bounds__(k45::kThreads) k45_select_inject(const __grid_constant__ k4::Params p,
-                                                                   const __grid_constant__ k5::Params sp) {
-    __shared__ int warp_cnt[k45::kThreads / 32];
-    __shared__ const uint4* rows[LOOKME_MAX_TOP_K];
-    __shared__ float w[LOOKME_MAX_TOP_K];
-    pdl_trigger();
-    pdl_wait();
-    const int64_t t = blockIdx.x;
-    const int tid = threadIdx.x;
+struct Seg {
+    int64_t b, len, r;
+};
+__device__ __forceinline__ Seg segment_of(const k5::Params& sp, int64_t t) {
     int lo = 0, hi = sp.n_seg;  // segment: off[lo] <= t < off[lo + 1]
     while (hi - lo > 1) {
         const int mid = (lo + hi) / 2;
         if (sp.off[mid] <= t) lo = mid;
         else hi = mid;
     }
-    const int64_t b = sp.off[lo], len = sp.off[lo + 1] - b;
-    const int64_t r = (int64_t)floor((double)len * sp.keep_ratio);
-    if (r <= 0) {
-        if (tid == 0 && sp.mask) sp.mask[t] = 0;
-        return;
+    Seg g;
+    g.b = sp.off[lo];
+    g.len = sp.off[lo + 1] - g.b;
+    g.r = (int64_t)floor((double)g.len * sp.keep_ratio);
+    return g;
+}
+}  // namespace k45
+
+template <typename T>
+__global__ void __launch_bounds__(k45::kThreads) k45_select_inject(const __grid_constant__ k4::Params p,
+                                                                   const __grid_constant__ k5::Params sp) {
+    using namespace k45;
+    __shared__ int warp_cnt[kTPC][kWarps];
+    __shared__ const uint4* rows[kTPC][LOOKME_MAX_TOP_K];
+    __shared__ float w[kTPC][LOOKME_MAX_TOP_K];
+    pdl_trigger();
+    pdl_wait();
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    int64_t t[kTPC];
+    Seg sg[kTPC];
+    bool valid[kTPC], ranked[kTPC];
+#pragma unroll
+    for (int u = 0; u < kTPC; ++u) {
+        t[u] = (int64_t)blockIdx.x * kTPC + u;
+        valid[u] = t[u] < p.N;
+        sg[u] = segment_of(sp, valid[u] ? t[u] : 0);
+        ranked[u] = valid[u] && sg[u].r > 0 && sg[u].r < sg[u].len;
     }
-    // Row addresses and weights (threads < top_k) and the first pass of
-    // priorities are independent loads, in flight together.
+    // Row addresses and weights: threads [64 u, 64 u + top_k) for token u.
+    const int u_row = tid / LOOKME_MAX_TOP_K, j_row = tid % LOOKME_MAX_TOP_K;
+    const bool row_thread = u_row < kTPC && j_row < p.top_k && (u_row == 0 ? valid[0] : valid[1]);
     int32_t sc = 0, pj = 0;
     float wj = 0.f;
-    if (tid < p.top_k) {
-        sc = p.scene[t];
-        pj = p.prim[t * p.top_k + tid];
-        wj = p.weight[t * p.top_k + tid];
+    if (row_thread) {
+        const int64_t tr = u_row == 0 ? t[0] : t[1];
+        sc = p.scene[tr];
+        pj = p.prim[tr * p.top_k + j_row];
+        wj = p.weight[tr * p.top_k + j_row];
     }
-    bool keep = true;
-    if (r < len) {
-        const float* pb = sp.priority + b;
-        const uint32_t kt = k5::prio_key(sp.priority[t]);
-        const int64_t tl = t - b;
-        int cnt = 0;
-        for (int64_t j0 = tid; j0 < len; j0 += k45::kUnroll * k45::kThreads) {
-            float v[k45::kUnroll];
+    // Ranks: one pass over the segment when both tokens share it (the usual
+    // case), else one pass per token.
+    int cnt[kTPC] = {};
+    uint32_t kt[kTPC];
 #pragma unroll
-            for (int u = 0; u < k45::kUnroll; ++u) {
-                const int64_t j = j0 + u * k45::kThreads;
-                v[u] = j < len ? pb[j] : 0.f;
+    for (int u = 0; u < kTPC; ++u) kt[u] = ranked[u] ? k5::prio_key(sp.priority[t[u]]) : 0u;
+    const bool shared_seg = ranked[0] && ranked[1] && sg[0].b == sg[1].b;
+#pragma unroll
+    for (int u = 0; u < kTPC; ++u) {
+        if (!ranked[u] || (u == 1 && shared_seg)) continue;
+        const float* pb = sp.priority + sg[u].b;
+        const int64_t len = sg[u].len;
+        for (int64_t j0 = tid; j0 < len; j0 += kUnroll * kThreads) {
+            float v[kUnroll];
+#pragma unroll
+            for (int q = 0; q < kUnroll; ++q) {
+                const int64_t j = j0 + q * kThreads;
+                v[q] = j < len ? pb[j] : 0.f;
             }
 #pragma unroll
-            for (int u = 0; u < k45::kUnroll; ++u) {
-                const int64_t j = j0 + u * k45::kThreads;
-                const uint32_t kj = k5::prio_key(v[u]);
-                cnt += j < len && ((kj > kt) || (kj == kt && j < tl));
+            for (int q = 0; q < kUnroll; ++q) {
+                const int64_t j = sg[u].b + j0 + q * kThreads;
+                const uint32_t kj = k5::prio_key(v[q]);
+                const bool in = j0 + q * kThreads < len;
+                cnt[u] += in && ((kj > kt[u]) || (kj == kt[u] && j < t[u]));
+                if (u == 0 && shared_seg) cnt[1] += in && ((kj > kt[1]) || (kj == kt[1] && j < t[1]));
             }
         }
-#pragma unroll
-        for (int o = 16; o; o >>= 1) cnt += __shfl_xor_sync(0xFFFFFFFFu, cnt, o);
-        if ((tid & 31) == 0) warp_cnt[tid / 32] = cnt;
     }
-    if (tid < p.top_k) {
+#pragma unroll
+    for (int u = 0; u < kTPC; ++u) {
+#pragma unroll
+        for (int o = 16; o; o >>= 1) cnt[u] += __shfl_xor_sync(0xFFFFFFFFu, cnt[u], o);
+        if (lane == 0) warp_cnt[u][warp] = cnt[u];
+    }
+    if (row_thread) {
         const int64_t s = min(max((int64_t)sc, (int64_t)0), p.S - 1);
         const int64_t pr = min(max((int64_t)pj, (int64_t)0), p.P - 1);
-        rows[tid] = reinterpret_cast<const uint4*>(reinterpret_cast<const T*>(p.values) + (s * p.P + pr) * p.dv);
-        w[tid] = wj;
+        rows[u_row][j_row] = reinterpret_cast<const uint4*>(reinterpret_cast<const T*>(p.values) + (s * p.P + pr) * p.dv);
+        w[u_row][j_row] = wj;
     }
     __syncthreads();  // counts, row addresses and weights visible to every thread
-    if (r < len) {
-        int total = 0;
 #pragma unroll
-        for (int i = 0; i < k45::kThreads / 32; ++i) total += warp_cnt[i];
-        keep = total < r;
+    for (int u = 0; u < kTPC; ++u) {
+        if (!valid[u]) continue;
+        bool keep = sg[u].r >= sg[u].len;
+        if (ranked[u]) {
+            int total = 0;
+#pragma unroll
+            for (int i = 0; i < kWarps; ++i) total += warp_cnt[u][i];
+            keep = total < sg[u].r;
+        }
+        if (tid == 0 && sp.mask) sp.mask[t[u]] = (uint8_t)keep;
+        if (keep) accumulate_store<T>(p, t[u], rows[u], w[u]);
     }
-    if (tid == 0 && sp.mask) sp.mask[t] = (uint8_t)keep;
-    if (keep) accumulate_store<T>(p, t, rows, w);
 }
 
 cudaError_t launch_select_inject(const LaunchCtx& c, const InjectArgs& a, const float* priority,
@@ -351,10 +388,10 @@ cudaError_t launch_select_inject(const LaunchCtx& c, const InjectArgs& a, const 
     sp.keep_ratio = keep_ratio;
     sp.n_seg = n_seg;
     for (int i = 0; i <= n_seg; ++i) sp.off[i] = seg_off_host ? seg_off_host[i] : (i == 0 ? 0 : a.N);
+    const unsigned grid = (unsigned)((a.N + k45::kTPC - 1) / k45::kTPC);
     if (a.dtype == LOOKME_BF16)
-        return launch_pdl(k45_select_inject<__nv_bfloat16>, dim3((unsigned)a.N), dim3(k45::kThreads), 0, c.stream,
-                          p, sp);
-    return launch_pdl(k45_select_inject<float>, dim3((unsigned)a.N), dim3(k45::kThreads), 0, c.stream, p, sp);
+        return launch_pdl(k45_select_inject<__nv_bfloat16>, dim3(grid), dim3(k45::kThreads), 0, c.stream, p, sp);
+    return launch_pdl(k45_select_inject<float>, dim3(grid), dim3(k45::kThreads), 0, c.stream, p, sp);
 }
 
 cudaError_t launch_inject(const LaunchCtx& c, const InjectArgs& a) {

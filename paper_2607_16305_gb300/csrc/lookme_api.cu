@@ -484,8 +484,15 @@ lookme_status lookme_load_scenes(lookme_table* t, int64_t scene_begin, int64_t n
     return LOOKME_OK;
 }
 
-lookme_status lookme_lookup(lookme_table* t, const void* queries, int64_t N, int32_t top_k, int32_t* scene_out,
-                            int32_t* prim_out, float* weight_out, float* qnorm_out, lookme_stream stream) {
+}  // extern "C"
+
+namespace {
+
+// lookme_lookup; with gate (tcgen05 level 2 only) the level-2 kernel also
+// computes the injection gate.
+lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32_t top_k, int32_t* scene_out,
+                          int32_t* prim_out, float* weight_out, float* qnorm_out, lookme_stream stream,
+                          const GateSpec* gate) {
     lookme_status st = check_table(t);
     if (st != LOOKME_OK) return st;
     const lookme_table_desc& d = t->d;
@@ -557,18 +564,21 @@ lookme_status lookme_lookup(lookme_table* t, const void* queries, int64_t N, int
     a.weight_out = weight_out;
     a.status = t->status;
     st = launch(t, s, KID_SCORE,
-                [&] { return t->tc_score ? launch_score_tc(ctx, a.keys, a) : launch_score(ctx, a); });
+                [&] { return t->tc_score ? launch_score_tc(ctx, a.keys, a, gate) : launch_score(ctx, a); });
     if (st != LOOKME_OK) return st;
     t->last_tokens = N;
     return LOOKME_OK;
 }
 
-lookme_status lookme_inject(lookme_table* t, const int32_t* scene, const int32_t* prim, const float* weight,
-                            int64_t N, int32_t top_k, const float* priority, const int64_t* seg_offsets,
-                            int32_t n_seg, double keep_ratio, void* const* hidden, int32_t n_layers,
-                            uint8_t* mask_out, int32_t* sel_out, lookme_stream stream) {
-    lookme_status st = check_table(t);
-    if (st != LOOKME_OK) return st;
+// Validated injection arguments: segment offsets (host), kept count, longest segment.
+struct InjectPlan {
+    std::vector<int64_t> off;
+    int n_seg = 1;
+    int64_t n_sel = 0, max_seg = 0;
+};
+
+lookme_status plan_inject(const lookme_table* t, int64_t N, int32_t top_k, const int64_t* seg_offsets, int32_t n_seg,
+                          double keep_ratio, void* const* hidden, int32_t n_layers, InjectPlan& plan) {
     const lookme_table_desc& d = t->d;
     if (N < 0 || N > INT32_MAX / 2) return fail(LOOKME_ERR_INVALID_ARG, "n_tokens %lld out of range", (long long)N);
     if (top_k < 1 || top_k > LOOKME_MAX_TOP_K || top_k > d.n_prims)
@@ -581,35 +591,32 @@ lookme_status lookme_inject(lookme_table* t, const int32_t* scene, const int32_t
         if (N > 0 && (!hidden[l] || !aligned16(hidden[l])))
             return fail(LOOKME_ERR_INVALID_ARG, "hidden[%d] is NULL or not 16-byte aligned", l);
     }
-    std::vector<int64_t> off;
     if (seg_offsets) {
         if (n_seg < 1 || n_seg > LOOKME_MAX_SEGMENTS)
             return fail(LOOKME_ERR_INVALID_ARG, "n_seg %d outside [1, %d]", n_seg, LOOKME_MAX_SEGMENTS);
-        off.assign(seg_offsets, seg_offsets + n_seg + 1);
-        if (off[0] != 0 || off[n_seg] != N)
+        plan.off.assign(seg_offsets, seg_offsets + n_seg + 1);
+        if (plan.off[0] != 0 || plan.off[n_seg] != N)
             return fail(LOOKME_ERR_INVALID_ARG, "seg_offsets must start at 0 and end at n_tokens");
         for (int i = 0; i < n_seg; ++i)
-            if (off[i + 1] < off[i]) return fail(LOOKME_ERR_INVALID_ARG, "seg_offsets must be non-decreasing");
+            if (plan.off[i + 1] < plan.off[i]) return fail(LOOKME_ERR_INVALID_ARG, "seg_offsets must be non-decreasing");
+        plan.n_seg = n_seg;
     } else {
-        n_seg = 1;
-        off = {0, N};
+        plan.n_seg = 1;
+        plan.off = {0, N};
     }
-    if (N == 0) return LOOKME_OK;
-    if (!scene || !prim || !weight) return fail(LOOKME_ERR_INVALID_ARG, "scene, prim and weight are required");
-    if (!priority && t->last_tokens != N)
-        return fail(LOOKME_ERR_STATE, "default priority needs a lookup of %lld tokens first", (long long)N);
-    int64_t n_sel = 0;
-    for (int i = 0; i < n_seg; ++i) n_sel += (int64_t)std::floor((double)(off[i + 1] - off[i]) * keep_ratio);
+    plan.n_sel = 0;
+    plan.max_seg = 0;
+    for (int i = 0; i < plan.n_seg; ++i) {
+        const int64_t len = plan.off[i + 1] - plan.off[i];
+        plan.n_sel += (int64_t)std::floor((double)len * keep_ratio);
+        plan.max_seg = std::max(plan.max_seg, len);
+    }
+    return LOOKME_OK;
+}
 
-    DeviceGuard guard(d.device);
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if ((st = ensure_scratch(t, N, s)) != LOOKME_OK) return st;
-    LaunchCtx ctx{s, t->num_sms};
-    uint8_t* mask = mask_out ? mask_out : t->mask;
-    int32_t* sel = sel_out ? sel_out : t->sel;
-    const float* pr = priority ? priority : t->qnorm;
-    int64_t max_seg = 0;
-    for (int i = 0; i < n_seg; ++i) max_seg = std::max(max_seg, off[i + 1] - off[i]);
+InjectArgs inject_args(const lookme_table* t, const int32_t* scene, const int32_t* prim, const float* weight,
+                       int64_t N, int32_t top_k, void* const* hidden, int32_t n_layers, int32_t* sel, int64_t n_sel) {
+    const lookme_table_desc& d = t->d;
     InjectArgs a;
     a.dtype = d.dtype;
     a.values = t->values;
@@ -625,14 +632,48 @@ lookme_status lookme_inject(lookme_table* t, const int32_t* scene, const int32_t
     a.S = d.n_scenes;
     a.n_layers = n_layers;
     for (int l = 0; l < n_layers; ++l) a.hidden[l] = hidden[l];
-    // Short segments and no kept-id list: selection fused into the injection.
-    if (!sel_out && max_seg <= kFusedMaxSegment)
-        return launch(t, s, KID_SELECT_INJECT, [&] {
-            return launch_select_inject(ctx, a, pr, off.data(), n_seg, keep_ratio, mask);
-        });
-    st = launch(t, s, KID_SELECT, [&] { return launch_select(ctx, pr, N, off.data(), n_seg, keep_ratio, mask, sel); });
+    return a;
+}
+
+}  // namespace
+
+extern "C" {
+
+lookme_status lookme_lookup(lookme_table* t, const void* queries, int64_t N, int32_t top_k, int32_t* scene_out,
+                            int32_t* prim_out, float* weight_out, float* qnorm_out, lookme_stream stream) {
+    return lookup_impl(t, queries, N, top_k, scene_out, prim_out, weight_out, qnorm_out, stream, nullptr);
+}
+
+lookme_status lookme_inject(lookme_table* t, const int32_t* scene, const int32_t* prim, const float* weight,
+                            int64_t N, int32_t top_k, const float* priority, const int64_t* seg_offsets,
+                            int32_t n_seg, double keep_ratio, void* const* hidden, int32_t n_layers,
+                            uint8_t* mask_out, int32_t* sel_out, lookme_stream stream) {
+    lookme_status st = check_table(t);
     if (st != LOOKME_OK) return st;
-    if (n_sel == 0) return LOOKME_OK;
+    InjectPlan plan;
+    if ((st = plan_inject(t, N, top_k, seg_offsets, n_seg, keep_ratio, hidden, n_layers, plan)) != LOOKME_OK) return st;
+    if (N == 0) return LOOKME_OK;
+    if (!scene || !prim || !weight) return fail(LOOKME_ERR_INVALID_ARG, "scene, prim and weight are required");
+    if (!priority && t->last_tokens != N)
+        return fail(LOOKME_ERR_STATE, "default priority needs a lookup of %lld tokens first", (long long)N);
+
+    DeviceGuard guard(t->d.device);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if ((st = ensure_scratch(t, N, s)) != LOOKME_OK) return st;
+    LaunchCtx ctx{s, t->num_sms};
+    uint8_t* mask = mask_out ? mask_out : t->mask;
+    int32_t* sel = sel_out ? sel_out : t->sel;
+    const float* pr = priority ? priority : t->qnorm;
+    const InjectArgs a = inject_args(t, scene, prim, weight, N, top_k, hidden, n_layers, sel, plan.n_sel);
+    // Short segments and no kept-id list: selection fused into the injection.
+    if (!sel_out && plan.max_seg <= kFusedMaxSegment)
+        return launch(t, s, KID_SELECT_INJECT, [&] {
+            return launch_select_inject(ctx, a, pr, plan.off.data(), plan.n_seg, keep_ratio, mask);
+        });
+    st = launch(t, s, KID_SELECT,
+                [&] { return launch_select(ctx, pr, N, plan.off.data(), plan.n_seg, keep_ratio, mask, sel); });
+    if (st != LOOKME_OK) return st;
+    if (plan.n_sel == 0) return LOOKME_OK;
     return launch(t, s, KID_INJECT, [&] { return launch_inject(ctx, a); });
 }
 
@@ -640,12 +681,49 @@ lookme_status lookme_lookup_inject(lookme_table* t, const void* queries, int64_t
                                    const float* priority, const int64_t* seg_offsets, int32_t n_seg,
                                    double keep_ratio, void* const* hidden, int32_t n_layers, int32_t* scene_out,
                                    int32_t* prim_out, float* weight_out, uint8_t* mask_out, lookme_stream stream) {
-    // The lookup's outputs feed the injection on the same stream; with PDL the
-    // injection kernel's launch overlaps the tail of the level-2 kernel.
-    lookme_status st = lookme_lookup(t, queries, N, top_k, scene_out, prim_out, weight_out, nullptr, stream);
+    lookme_status st = check_table(t);
     if (st != LOOKME_OK) return st;
-    return lookme_inject(t, scene_out, prim_out, weight_out, N, top_k, priority, seg_offsets, n_seg, keep_ratio,
-                         hidden, n_layers, mask_out, nullptr, stream);
+    InjectPlan plan;
+    if ((st = plan_inject(t, N, top_k, seg_offsets, n_seg, keep_ratio, hidden, n_layers, plan)) != LOOKME_OK) return st;
+    const bool gate_in_lookup =
+        t->tc_score && N > 0 && plan.n_seg <= kMaxGateSegments && plan.max_seg <= kFusedMaxSegment;
+    if (!gate_in_lookup) {
+        // The two calls in sequence; with PDL the injection kernel's launch
+        // overlaps the tail of the level-2 kernel.
+        st = lookme_lookup(t, queries, N, top_k, scene_out, prim_out, weight_out, nullptr, stream);
+        if (st != LOOKME_OK) return st;
+        return lookme_inject(t, scene_out, prim_out, weight_out, N, top_k, priority, seg_offsets, n_seg, keep_ratio,
+                             hidden, n_layers, mask_out, nullptr, stream);
+    }
+    // The level-2 kernel decides the gate (its warps are idle until the first
+    // keys land) and lists the kept tokens; the injection then runs on the
+    // kept tokens only.
+    DeviceGuard guard(t->d.device);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if ((st = ensure_scratch(t, N, s)) != LOOKME_OK) return st;
+    GateSpec gs;
+    memset(&gs, 0, sizeof(gs));
+    gs.enabled = 1;
+    gs.n_seg = plan.n_seg;
+    gs.N = N;
+    gs.keep_ratio = keep_ratio;
+    gs.priority = priority ? priority : t->qnorm;
+    gs.mask = mask_out ? mask_out : t->mask;
+    gs.sel = t->sel;
+    int64_t base = 0;
+    for (int i = 0; i < plan.n_seg; ++i) {
+        gs.off[i] = plan.off[i];
+        gs.sel_base[i] = base;
+        base += (int64_t)std::floor((double)(plan.off[i + 1] - plan.off[i]) * keep_ratio);
+    }
+    gs.off[plan.n_seg] = plan.off[plan.n_seg];
+    st = lookup_impl(t, queries, N, top_k, scene_out, prim_out, weight_out, nullptr, stream, &gs);
+    if (st != LOOKME_OK) return st;
+    if (plan.n_sel == 0) return LOOKME_OK;
+    LaunchCtx ctx{s, t->num_sms};
+    const InjectArgs a =
+        inject_args(t, scene_out, prim_out, weight_out, N, top_k, hidden, n_layers, t->sel, plan.n_sel);
+    return launch(t, s, KID_INJECT, [&] { return launch_inject(ctx, a); });
 }
 
 lookme_status lookme_last_lookup_stats(lookme_table* t, lookme_lookup_stats* out, lookme_stream stream) {
