@@ -165,8 +165,8 @@ lookme_status lookme_inject(lookme_table* table, const int32_t* scene, const int
  * the same results (Sec. "Hierarchical Lookup" then Sec. "Sparse Injection").
  * The arguments mean what they mean there; priority NULL = the query norms of
  * these queries; mask_out (device [n_tokens] uint8, or NULL) receives the
- * gate.  On tensor-core tables with at most 64 segments of at most 8,192
- * tokens, the level-2 kernel decides the gate itself and the injection visits
+ * gate.  With at most 64 segments of at most 8,192 tokens, the gate is
+ * decided during the lookup (beside the bucketing) and the injection visits
  * only the kept tokens.  Errors: those of lookme_lookup and lookme_inject
  * (the injection arguments are checked before anything runs). */
 lookme_status lookme_lookup_inject(lookme_table* table, const void* queries, int64_t n_tokens, int32_t top_k,

@@ -144,8 +144,11 @@ cudaError_t launch_route_simt(const LaunchCtx& c, int dtype, const void* q, cons
                               unsigned long long* best);
 // K2 (also resets best[0, N) to 0 for the next call)
 constexpr int kTokensPerItem = 8;
+// gate (optional, GateSpec declared below) adds CTAs that compute the injection gate.
+struct GateSpec;
 cudaError_t launch_bucket(const LaunchCtx& c, unsigned long long* best, int64_t N, int64_t S,
-                          int32_t* scene_out, int32_t* perm, WorkItem* work, int32_t* routed, int32_t* counters);
+                          int32_t* scene_out, int32_t* perm, WorkItem* work, int32_t* routed, int32_t* counters,
+                          const GateSpec* gate = nullptr);
 // K3
 struct ScoreArgs {
     int dtype;
@@ -166,10 +169,10 @@ struct ScoreArgs {
 cudaError_t launch_score(const LaunchCtx& c, const ScoreArgs& a);
 // Whether the level-2 kernel's shared-memory plan fits this table shape.
 bool score_shape_supported(int dtype, int64_t P, int dk);
-// The injection gate computed inside the tcgen05 level-2 kernel (by warps
-// that would otherwise wait for the first keys): token t of segment s is kept
-// iff its rank (larger priority first, lower index on ties) is below
-// r_s = floor(len_s * keep_ratio); kept tokens go to sel[sel_base[s] + rank].
+// The injection gate computed by extra CTAs of the bucketing kernel: token t
+// of segment s is kept iff its rank (larger priority first, lower index on
+// ties) is below r_s = floor(len_s * keep_ratio); kept tokens go to
+// sel[sel_base[s] + rank].
 constexpr int kMaxGateSegments = 64;
 struct GateSpec {
     int enabled;
@@ -186,9 +189,7 @@ struct GateSpec {
 // Level 2 on tcgen05 (bf16 tables).  keys_tiled holds every scene's (or
 // staging slot's) keys in the tiled layout of k_tile_keys, one block of
 // score_tc_block_bytes(P, d_k) bytes per scene; ScoreArgs::keys is unused.
-// gate (optional) adds the injection gate.
-cudaError_t launch_score_tc(const LaunchCtx& c, const void* keys_tiled, const ScoreArgs& a,
-                            const GateSpec* gate = nullptr);
+cudaError_t launch_score_tc(const LaunchCtx& c, const void* keys_tiled, const ScoreArgs& a);
 bool score_tc_shape_supported(int64_t P, int dk);
 int64_t score_tc_block_bytes(int64_t P, int dk);
 // Load time: rewrites n scenes of row-major keys [n][P][d_k] (bf16, device

@@ -12,13 +12,85 @@
 //                  position in it is its `slot`
 //   counters[0..3] number of work items, of routed scenes, largest bucket;
 //                  [3] is reset to 0 for the level-2 kernel's work taking
+//
+// With a gate, CTAs 1.. compute the injection gate meanwhile, eight tokens
+// per CTA (one per warp; a light load per SM so they finish within the
+// bucketing): rank_t = #{ j in segment : pi_j > pi_t, or pi_j == pi_t and
+// j < t }, kept iff rank_t < r, the kept ones listed at sel[sel_base + rank_t].
+// Each CTA stages the priorities its tokens' segments span in shared memory
+// once.  This runs before the level-2 key stream, whose copies would
+// otherwise queue every small load behind them.
+#include <string.h>
+
+#include <algorithm>
+
 #include "common.cuh"
 
 namespace lookme {
 
 namespace {
 constexpr int kThreads = 1024;
+constexpr int kGateTokens = 8;     // tokens per gate CTA
+constexpr int kGateStage = 32768;  // bytes of priorities a gate CTA stages
 
+__device__ __forceinline__ int segment_index(const GateSpec& gs, int64_t t) {
+    int lo = 0, hi = gs.n_seg;  // off[lo] <= t < off[lo + 1]
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) / 2;
+        if (gs.off[mid] <= t) lo = mid;
+        else hi = mid;
+    }
+    return lo;
+}
+
+__device__ void gate_block(const GateSpec& gs, float* buf, int cap) {
+    const int tid = threadIdx.x, warp = tid / 32, lane = tid % 32;
+    const int64_t tb = (int64_t)(blockIdx.x - 1) * kGateTokens, te = min(gs.N, tb + kGateTokens);
+    if (tb >= te) return;  // uniform for the CTA
+    const int64_t rb = gs.off[segment_index(gs, tb)], re = gs.off[segment_index(gs, te - 1) + 1];
+    const bool staged = re - rb <= cap;  // uniform for the CTA
+    if (staged) {
+        for (int64_t i = tid; i < re - rb; i += kThreads) buf[i] = gs.priority[rb + i];
+        __syncthreads();
+    }
+    const int64_t t = tb + warp;
+    if (warp >= kGateTokens || t >= te) return;
+    const int sg = segment_index(gs, t);
+    const int64_t b = gs.off[sg], len = gs.off[sg + 1] - b;
+    const int64_t r = (int64_t)floor((double)len * gs.keep_ratio);
+    bool keep;
+    int64_t rank = t - b;  // the slot when every token of the segment is kept
+    if (r <= 0) {
+        keep = false;
+    } else if (r >= len) {
+        keep = true;
+    } else {
+        const uint32_t kt = orderable(gs.priority[t]);
+        const int tl = (int)(t - b);
+        const float* src = staged ? buf + (b - rb) : gs.priority + b;
+        int cnt = 0;
+        const int n = (int)len;
+        int i = lane;
+        for (; i + 96 < n; i += 128) {
+            const float v0 = src[i], v1 = src[i + 32], v2 = src[i + 64], v3 = src[i + 96];
+            const uint32_t k0 = orderable(v0), k1 = orderable(v1), k2 = orderable(v2), k3 = orderable(v3);
+            cnt += ((k0 > kt) || (k0 == kt && i < tl)) + ((k1 > kt) || (k1 == kt && i + 32 < tl)) +
+                   ((k2 > kt) || (k2 == kt && i + 64 < tl)) + ((k3 > kt) || (k3 == kt && i + 96 < tl));
+        }
+        for (; i < n; i += 32) {
+            const uint32_t kj = orderable(src[i]);
+            cnt += (kj > kt) || (kj == kt && i < tl);
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) cnt += __shfl_xor_sync(0xFFFFFFFFu, cnt, o);
+        rank = cnt;
+        keep = rank < r;
+    }
+    if (lane == 0) {
+        gs.mask[t] = (uint8_t)keep;
+        if (keep) gs.sel[gs.sel_base[sg] + rank] = (int32_t)t;
+    }
+}
 // Exclusive block-wide scan of three counters at once.
 __device__ void block_exclusive_scan3(int3 v, int3& excl, int3& total, int3* warp_buf) {
     const int lane = threadIdx.x % 32, warp = threadIdx.x / 32;
@@ -63,12 +135,16 @@ __device__ void block_exclusive_scan3(int3 v, int3& excl, int3& total, int3* war
 __global__ void __launch_bounds__(kThreads, 1)
     k2_bucket(unsigned long long* __restrict__ best, int64_t N, int S, int32_t* __restrict__ scene_out,
               int32_t* __restrict__ perm, WorkItem* __restrict__ work, int32_t* __restrict__ routed,
-              int32_t* __restrict__ counters) {
-    extern __shared__ int cnt[];  // [S]: counts, then running token offsets
+              int32_t* __restrict__ counters, const __grid_constant__ GateSpec gate, int smem_bytes) {
+    extern __shared__ int cnt[];  // CTA 0: [S] counts, then running token offsets; gate CTAs: priorities
     __shared__ int3 warp_buf[33];
     __shared__ int max_bucket;
     pdl_trigger();
     pdl_wait();
+    if (blockIdx.x > 0) {
+        gate_block(gate, reinterpret_cast<float*>(cnt), smem_bytes / 4);
+        return;
+    }
     const int tid = threadIdx.x;
     for (int s = tid; s < S; s += kThreads) cnt[s] = 0;
     if (tid == 0) max_bucket = 0;
@@ -130,15 +206,23 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 cudaError_t launch_bucket(const LaunchCtx& c, unsigned long long* best, int64_t N, int64_t S,
-                          int32_t* scene_out, int32_t* perm, WorkItem* work, int32_t* routed, int32_t* counters) {
-    const size_t smem = (size_t)S * sizeof(int);
-    return launch_pdl(k2_bucket, dim3(1), dim3(kThreads), smem, c.stream, best, N, (int)S, scene_out, perm, work,
-                      routed, counters);
+                          int32_t* scene_out, int32_t* perm, WorkItem* work, int32_t* routed, int32_t* counters,
+                          const GateSpec* gate) {
+    GateSpec gs;
+    if (gate) {
+        gs = *gate;
+    } else {
+        memset(&gs, 0, sizeof(gs));
+    }
+    const int gate_ctas = gate ? (int)((N + kGateTokens - 1) / kGateTokens) : 0;
+    const int smem = (int)std::max<int64_t>(S * (int64_t)sizeof(int), gate ? kGateStage : 0);
+    return launch_pdl(k2_bucket, dim3(1 + gate_ctas), dim3(kThreads), (size_t)smem, c.stream, best, N, (int)S,
+                      scene_out, perm, work, routed, counters, gs, smem);
 }
 
 cudaError_t configure_bucket_kernel() {
     return cudaFuncSetAttribute(k2_bucket, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)(LOOKME_MAX_SCENES * sizeof(int)));
+                                (int)std::max<int64_t>(LOOKME_MAX_SCENES * sizeof(int), kGateStage));
 }
 
 }  // namespace lookme

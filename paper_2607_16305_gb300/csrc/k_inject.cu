@@ -11,11 +11,12 @@
 //   layer l sharing the table, rounded once to the hidden dtype.  Rows that are
 //   not kept are never touched.
 #include "common.cuh"
+#include "select.cuh"
 
 namespace lookme {
 
 namespace k5 {
-constexpr int kThreads = 1024;
+constexpr int kThreads = sel::kSelectThreads;
 
 struct Params {
     const float* priority;
@@ -28,42 +29,9 @@ struct Params {
 
 __device__ __forceinline__ uint32_t prio_key(float f) { return orderable(f); }
 
-// Block-wide exclusive scan of one int (1024 threads).
-__device__ int block_excl_scan(int v, int& total, int* buf) {
-    const int lane = threadIdx.x % 32, warp = threadIdx.x / 32;
-    int inc = v;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int n = __shfl_up_sync(0xFFFFFFFFu, inc, o);
-        if (lane >= o) inc += n;
-    }
-    if (lane == 31) buf[warp] = inc;
-    __syncthreads();
-    if (warp == 0) {
-        const int w = buf[lane];
-        int wi = w;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int n = __shfl_up_sync(0xFFFFFFFFu, wi, o);
-            if (lane >= o) wi += n;
-        }
-        buf[lane] = wi - w;
-        if (lane == 31) buf[32] = wi;
-    }
-    __syncthreads();
-    const int r = buf[warp] + inc - v;
-    total = buf[32];
-    __syncthreads();
-    return r;
-}
 }  // namespace k5
 
 __global__ void __launch_bounds__(k5::kThreads, 1) k5_select(const __grid_constant__ k5::Params p) {
-    using namespace k5;
-    __shared__ int hist[256];
-    __shared__ int scan_buf[33];
-    __shared__ uint32_t sh_prefix;
-    __shared__ int sh_remaining;
     pdl_trigger();
     pdl_wait();
     const int seg = blockIdx.x;
@@ -71,79 +39,7 @@ __global__ void __launch_bounds__(k5::kThreads, 1) k5_select(const __grid_consta
     const int64_t r = (int64_t)floor((double)len * p.keep_ratio);
     int64_t sel_base = 0;
     for (int i = 0; i < seg; ++i) sel_base += (int64_t)floor((double)(p.off[i + 1] - p.off[i]) * p.keep_ratio);
-    const int tid = threadIdx.x;
-
-    uint32_t prefix = 0, pmask = 0;
-    int remaining = (int)r;
-    if (r > 0 && r < len) {
-        for (int shift = 24; shift >= 0; shift -= 8) {
-            for (int i = tid; i < 256; i += kThreads) hist[i] = 0;
-            __syncthreads();
-            for (int64_t i = tid; i < len; i += kThreads) {
-                const uint32_t k = prio_key(p.priority[b + i]);
-                if ((k & pmask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1);
-            }
-            __syncthreads();
-            // One warp finds the digit holding the r-th largest key: lane l
-            // owns bins 255 - 8 l ... 248 - 8 l (descending), an exclusive
-            // prefix over lanes gives the count above each lane's bins.
-            if (tid < 32) {
-                const int top = 255 - 8 * tid;
-                int local = 0;
-#pragma unroll
-                for (int i = 0; i < 8; ++i) local += hist[top - i];
-                int inc = local;
-#pragma unroll
-                for (int o = 1; o < 32; o <<= 1) {
-                    const int n = __shfl_up_sync(0xFFFFFFFFu, inc, o);
-                    if (tid >= o) inc += n;
-                }
-                const int excl = inc - local;
-                if (excl < remaining && remaining <= inc) {
-                    int above = excl, d = top;
-                    for (int i = 0; i < 8; ++i) {
-                        d = top - i;
-                        if (above + hist[d] >= remaining) break;
-                        above += hist[d];
-                    }
-                    sh_prefix = prefix | ((uint32_t)d << shift);
-                    sh_remaining = remaining - above;
-                }
-            }
-            __syncthreads();
-            prefix = sh_prefix;
-            remaining = sh_remaining;
-            pmask |= 255u << shift;
-            __syncthreads();
-        }
-    }
-    // Keep: key > threshold, or key == threshold among the first `remaining` in token order.
-    const uint32_t thr = prefix;
-    int eq_seen = 0, kept_seen = 0;
-    for (int64_t i0 = 0; i0 < len; i0 += kThreads) {
-        const int64_t i = i0 + tid;
-        int is_eq = 0, keep = 0;
-        if (i < len) {
-            if (r >= len) {
-                keep = 1;
-            } else if (r > 0) {
-                const uint32_t k = prio_key(p.priority[b + i]);
-                keep = k > thr;
-                is_eq = k == thr;
-            }
-        }
-        int eq_total;
-        const int eq_rank = block_excl_scan(is_eq, eq_total, scan_buf);
-        if (is_eq && eq_seen + eq_rank < remaining) keep = 1;
-        int kept_total;
-        const int kept_rank = block_excl_scan(keep, kept_total, scan_buf);
-        if (i < len) {
-            if (p.mask) p.mask[b + i] = (uint8_t)keep;
-            if (keep) p.sel[sel_base + kept_seen + kept_rank] = (int32_t)(b + i);
-        }
-        eq_seen += eq_total;
-        kept_seen += kept_total;
-    }
+    sel::select_segment(p.priority, b, len, r, sel_base, p.mask, p.sel);
 }
 
 cudaError_t launch_select(const LaunchCtx& c, const float* priority, int64_t N, const int64_t* seg_off_host,

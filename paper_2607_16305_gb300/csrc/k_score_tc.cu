@@ -176,52 +176,6 @@ __device__ __forceinline__ void topk_item(const float* z, int64_t P, int top_k, 
     else topk_large(z, P, top_k, lane, t, prim_out, weight_out);
 }
 
-// The injection gate of tokens [t0, t1), one token per warp (warp wid of nw):
-// rank_t = #{ j in segment : pi_j > pi_t, or pi_j == pi_t and j < t }, kept iff
-// rank_t < r; writes mask[t] and, for kept tokens, sel[sel_base + rank_t].
-__device__ void gate_tokens(const GateSpec& gs, int64_t t0, int64_t t1, int wid, int nw, int lane) {
-    constexpr int U = 16;  // priorities in flight per lane (a 1,024-token segment in two passes)
-    for (int64_t t = t0 + wid; t < t1; t += nw) {
-        int lo = 0, hi = gs.n_seg;
-        while (hi - lo > 1) {
-            const int mid = (lo + hi) / 2;
-            if (gs.off[mid] <= t) lo = mid;
-            else hi = mid;
-        }
-        const int64_t b = gs.off[lo], len = gs.off[lo + 1] - b;
-        const int64_t r = (int64_t)floor((double)len * gs.keep_ratio);
-        bool keep;
-        int64_t rank = t - b;  // the slot when every token of the segment is kept
-        if (r <= 0) {
-            keep = false;
-        } else if (r >= len) {
-            keep = true;
-        } else {
-            const uint32_t kt = orderable(gs.priority[t]);
-            const float* pb = gs.priority + b;
-            int cnt = 0;
-            for (int64_t j0 = lane; j0 < len; j0 += 32 * U) {
-                float v[U];
-#pragma unroll
-                for (int u = 0; u < U; ++u) v[u] = j0 + 32 * u < len ? pb[j0 + 32 * u] : 0.f;
-#pragma unroll
-                for (int u = 0; u < U; ++u) {
-                    const int64_t j = j0 + 32 * u;
-                    const uint32_t kj = orderable(v[u]);
-                    cnt += j < len && ((kj > kt) || (kj == kt && b + j < t));
-                }
-            }
-#pragma unroll
-            for (int o = 16; o; o >>= 1) cnt += __shfl_xor_sync(0xFFFFFFFFu, cnt, o);
-            rank = cnt;
-            keep = rank < r;
-        }
-        if (lane == 0) {
-            gs.mask[t] = (uint8_t)keep;
-            if (keep) gs.sel[gs.sel_base[lo] + rank] = (int32_t)t;
-        }
-    }
-}
 }  // namespace k3tc
 
 __global__ void __launch_bounds__(k3tc::kThreads, 1)
@@ -229,7 +183,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
                 int64_t P, int dk, int top_k, float scale, const WorkItem* __restrict__ work,
                 const int32_t* __restrict__ counters, const int32_t* __restrict__ perm, int use_slots,
                 int32_t* __restrict__ prim_out, float* __restrict__ weight_out, uint32_t* __restrict__ status,
-                const __grid_constant__ k3tc::Geometry g, const __grid_constant__ GateSpec gate) {
+                const __grid_constant__ k3tc::Geometry g) {
     using namespace k3tc;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -264,13 +218,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
     const int n_work = counters[0];
     const int G = gridDim.x;
     const int my_items = n_work > (int)blockIdx.x ? (n_work - (int)blockIdx.x + G - 1) / G : 0;
-    // This CTA's share of the injection gate (a contiguous token range).
-    const int64_t gate_per = gate.enabled ? (gate.N + G - 1) / G : 0;
-    const int64_t gate_t0 = min((int64_t)blockIdx.x * gate_per, gate.N), gate_t1 = min(gate_t0 + gate_per, gate.N);
-    if (my_items == 0) {  // uniform for the CTA: nothing allocated yet
-        if (gate.enabled) k3tc::gate_tokens(gate, gate_t0, gate_t1, warp, kThreads / 32, lane);
-        return;
-    }
+    if (my_items == 0) return;  // uniform for the CTA: nothing allocated yet
     auto item_index = [&](int i) { return (int)blockIdx.x + i * G; };
     // N-tile nt: its first sub-block, its sub-block count (1 or 2) and its N.
     auto nt_base = [&](int nt) { return nt * 2 * g.nkb; };
@@ -413,8 +361,6 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         const int eg = e % kGroupWarps;   // token of the top-k, column slice of the read-out
         const int quarter = warp & 3;     // TMEM lanes this warp may access
         float* zg = zs + grp * (g.zbytes / 4);
-        // The gate first: the first keys are microseconds away.
-        if (gate.enabled) k3tc::gate_tokens(gate, gate_t0, gate_t1, e, kEpiWarps, lane);
         for (int i = grp; i < my_items; i += 2) {
             const int ms = i % kISlots;
             bool ok = __all_sync(0xFFFFFFFFu, ptx::mbar_wait(&ifull[ms], (i / kISlots) & 1, abort, kTimeoutNs));
@@ -533,19 +479,13 @@ int64_t score_tc_block_bytes(int64_t P, int dk) {
     return (int64_t)g.spi * k3tc::kSubBytes;
 }
 
-cudaError_t launch_score_tc(const LaunchCtx& c, const void* keys_tiled, const ScoreArgs& a, const GateSpec* gate) {
+cudaError_t launch_score_tc(const LaunchCtx& c, const void* keys_tiled, const ScoreArgs& a) {
     const k3tc::Geometry g = k3tc::geometry(a.P, a.dk);
     if (!score_tc_shape_supported(a.P, a.dk)) return cudaErrorInvalidConfiguration;
-    GateSpec gs;
-    if (gate) {
-        gs = *gate;
-    } else {
-        memset(&gs, 0, sizeof(gs));
-    }
     return launch_pdl(k3_score_tc, dim3(c.num_sms), dim3(k3tc::kThreads), (size_t)g.smem, c.stream,
                       (const uint8_t*)keys_tiled, (int64_t)g.spi * k3tc::kSubBytes, (const __nv_bfloat16*)a.q, a.P,
                       a.dk, a.top_k, a.scale, a.work, (const int32_t*)a.counters, a.perm, a.use_slots, a.prim_out,
-                      a.weight_out, a.status, g, gs);
+                      a.weight_out, a.status, g);
 }
 
 cudaError_t configure_score_tc_kernel() {

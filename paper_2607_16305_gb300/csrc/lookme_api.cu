@@ -488,8 +488,7 @@ lookme_status lookme_load_scenes(lookme_table* t, int64_t scene_begin, int64_t n
 
 namespace {
 
-// lookme_lookup; with gate (tcgen05 level 2 only) the level-2 kernel also
-// computes the injection gate.
+// lookme_lookup; with gate the bucketing kernel also computes the injection gate.
 lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32_t top_k, int32_t* scene_out,
                           int32_t* prim_out, float* weight_out, float* qnorm_out, lookme_stream stream,
                           const GateSpec* gate) {
@@ -538,7 +537,8 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
     }
     if (st != LOOKME_OK) return st;
     st = launch(t, s, KID_BUCKET, [&] {
-        return launch_bucket(ctx, t->best, N, d.n_scenes, scene_out, t->perm, t->work, t->routed, t->counters);
+        return launch_bucket(ctx, t->best, N, d.n_scenes, scene_out, t->perm, t->work, t->routed, t->counters,
+                             gate);
     });
     if (st != LOOKME_OK) return st;
     const bool staged = d.residency == LOOKME_RES_HOST_STAGED;
@@ -564,7 +564,7 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
     a.weight_out = weight_out;
     a.status = t->status;
     st = launch(t, s, KID_SCORE,
-                [&] { return t->tc_score ? launch_score_tc(ctx, a.keys, a, gate) : launch_score(ctx, a); });
+                [&] { return t->tc_score ? launch_score_tc(ctx, a.keys, a) : launch_score(ctx, a); });
     if (st != LOOKME_OK) return st;
     t->last_tokens = N;
     return LOOKME_OK;
@@ -685,8 +685,7 @@ lookme_status lookme_lookup_inject(lookme_table* t, const void* queries, int64_t
     if (st != LOOKME_OK) return st;
     InjectPlan plan;
     if ((st = plan_inject(t, N, top_k, seg_offsets, n_seg, keep_ratio, hidden, n_layers, plan)) != LOOKME_OK) return st;
-    const bool gate_in_lookup =
-        t->tc_score && N > 0 && plan.n_seg <= kMaxGateSegments && plan.max_seg <= kFusedMaxSegment;
+    const bool gate_in_lookup = N > 0 && plan.n_seg <= kMaxGateSegments && plan.max_seg <= kFusedMaxSegment;
     if (!gate_in_lookup) {
         // The two calls in sequence; with PDL the injection kernel's launch
         // overlaps the tail of the level-2 kernel.
@@ -695,9 +694,8 @@ lookme_status lookme_lookup_inject(lookme_table* t, const void* queries, int64_t
         return lookme_inject(t, scene_out, prim_out, weight_out, N, top_k, priority, seg_offsets, n_seg, keep_ratio,
                              hidden, n_layers, mask_out, nullptr, stream);
     }
-    // The level-2 kernel decides the gate (its warps are idle until the first
-    // keys land) and lists the kept tokens; the injection then runs on the
-    // kept tokens only.
+    // The bucketing kernel's extra CTAs decide the gate and list the kept
+    // tokens while it sorts; the injection then runs on the kept tokens only.
     DeviceGuard guard(t->d.device);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if ((st = ensure_scratch(t, N, s)) != LOOKME_OK) return st;
