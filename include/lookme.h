@@ -189,8 +189,9 @@ typedef struct {
 lookme_status lookme_last_lookup_stats(lookme_table* table, lookme_lookup_stats* out, lookme_stream stream);
 
 /* Device status word of the table (bit 0: a bounded wait inside a kernel
- * gave up; the kernel then skipped its remaining work).  Synchronises the
- * stream.  reset != 0 clears it afterwards. */
+ * gave up; the kernel then skipped its remaining work; bit 1: it was the
+ * level-1 kernel, bit 2: a level-2 kernel).  Synchronises the stream.
+ * reset != 0 clears it afterwards. */
 lookme_status lookme_device_status(lookme_table* table, uint32_t* status, int reset, lookme_stream stream);
 
 /* Number of CUDA kernels this table has launched since creation. */

@@ -32,6 +32,8 @@ enum KernelId : int32_t {
 
 // Device status bits (table status word).
 constexpr uint32_t STATUS_WAIT_TIMEOUT = 1u;
+constexpr uint32_t STATUS_IN_ROUTE = 2u;  // set with STATUS_WAIT_TIMEOUT by the level-1 kernel
+constexpr uint32_t STATUS_IN_SCORE = 4u;  // set with STATUS_WAIT_TIMEOUT by a level-2 kernel
 
 // ------------------------------------------------------------ element access
 __device__ __forceinline__ float to_f32(float x) { return x; }

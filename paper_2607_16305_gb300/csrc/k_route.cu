@@ -398,7 +398,7 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem_base, 2 * BN);
     }
-    if (threadIdx.x == 0 && *abort) atomicOr(status, STATUS_WAIT_TIMEOUT);
+    if (threadIdx.x == 0 && *abort) atomicOr(status, STATUS_WAIT_TIMEOUT | STATUS_IN_ROUTE);
 }
 
 template <int BN, int STAGES>
@@ -436,9 +436,14 @@ cudaError_t launch_route_tc(const LaunchCtx& c, const void* tmap_q, const void* 
     if (dk > kRouteTcMaxDk) return cudaErrorInvalidValue;
     const int m_tiles = (int)((N + k1tc::BM - 1) / k1tc::BM);
     // Narrow scene tiles when there are few token tiles, so more CTAs share the work.
-    if ((int64_t)m_tiles * ((S + 255) / 256) >= c.num_sms)
-        return launch_route_tc_t<256, 3>(c, tmap_q, tmap_c[2], N, S, dk, inv_cnorm, bias, qnorm, qnorm_out, best,
+    if ((int64_t)m_tiles * ((S + 255) / 256) >= c.num_sms) {
+        // Three centroid stages unless the token tile of a wide d_k leaves room for two only.
+        if (k1tc::smem_bytes(256, 3, (dk + k1tc::BK - 1) / k1tc::BK) <= 227 * 1024)
+            return launch_route_tc_t<256, 3>(c, tmap_q, tmap_c[2], N, S, dk, inv_cnorm, bias, qnorm, qnorm_out, best,
+                                              status);
+        return launch_route_tc_t<256, 2>(c, tmap_q, tmap_c[2], N, S, dk, inv_cnorm, bias, qnorm, qnorm_out, best,
                                           status);
+    }
     if ((int64_t)m_tiles * ((S + 127) / 128) >= c.num_sms)
         return launch_route_tc_t<128, 4>(c, tmap_q, tmap_c[1], N, S, dk, inv_cnorm, bias, qnorm, qnorm_out, best,
                                           status);
@@ -449,6 +454,8 @@ cudaError_t launch_route_tc(const LaunchCtx& c, const void* tmap_q, const void* 
 cudaError_t configure_route_kernels() {
     cudaError_t e;
     e = cudaFuncSetAttribute(k1_route_tc<256, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(k1_route_tc<256, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(k1_route_tc<128, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
     if (e != cudaSuccess) return e;

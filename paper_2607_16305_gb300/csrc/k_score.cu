@@ -252,7 +252,7 @@ __global__ void __launch_bounds__(k3::kThreads, 1)
                 if (s >= 0) ptx::mbar_wait_drain(&full[s % g.n_stages], (uint32_t)((s / g.n_stages) & 1), kTimeoutNs);
             for (uint32_t s = item_seq >= (uint32_t)g.n_items ? item_seq - g.n_items + 1 : 0; s <= item_seq; ++s)
                 ptx::mbar_wait_drain(&ifull[s % g.n_items], (s / g.n_items) & 1u, kTimeoutNs);
-            atomicOr(status, STATUS_WAIT_TIMEOUT);
+            atomicOr(status, STATUS_WAIT_TIMEOUT | STATUS_IN_SCORE);
         }
         return;
     }

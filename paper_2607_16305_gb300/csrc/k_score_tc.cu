@@ -114,7 +114,7 @@ inline Geometry geometry(int64_t P, int dk) {
     g.off_b = g.n_stages * g.slot_bytes;
     g.off_z = g.off_b + kBSlots * g.b_bytes;
     g.off_bar = g.off_z + 2 * g.zbytes;
-    g.off_meta = g.off_bar + (2 * kMaxStages + 2 * kBSlots + 2 * kISlots + 2 * 2 + 1) * 8;
+    g.off_meta = g.off_bar + (2 * kMaxStages + 2 * kBSlots + 2 * kISlots + 4 + 2 + 1) * 8;
     g.smem = g.off_meta + kISlots * ((int)sizeof(WorkItem) + kTok * 4) + 16 + 1024;
     return g;
 }
@@ -196,8 +196,12 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
     uint64_t* bempty = bfull + kBSlots;
     uint64_t* ifull = bempty + kBSlots;
     uint64_t* iempty = ifull + kISlots;
+    // D buffer b ready for epilogue group q: dready[2 q + b].  Each group waits
+    // only on its own pair, in the order the MMA commits to it, so no waiter is
+    // ever two phases behind a barrier (the two groups share both buffers when
+    // an item has several N-tiles).
     uint64_t* dready = iempty + kISlots;
-    uint64_t* tempty = dready + 2;
+    uint64_t* tempty = dready + 4;
     uint64_t* drain = tempty + 2;
     WorkItem* items = reinterpret_cast<WorkItem*>(smem + g.off_meta);
     int32_t* toks = reinterpret_cast<int32_t*>(items + kISlots);
@@ -241,10 +245,8 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             ptx::mbar_init(&ifull[i], 1);
             ptx::mbar_init(&iempty[i], kGroupWarps);
         }
-        for (int i = 0; i < 2; ++i) {
-            ptx::mbar_init(&dready[i], 1);
-            ptx::mbar_init(&tempty[i], kGroupWarps);
-        }
+        for (int i = 0; i < 4; ++i) ptx::mbar_init(&dready[i], 1);
+        for (int i = 0; i < 2; ++i) ptx::mbar_init(&tempty[i], kGroupWarps);
         ptx::mbar_init(drain, 1);
         *abort = 0;
         ptx::fence_mbar_init();
@@ -339,7 +341,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
                         mma_kblock(1u, d, ad0 + (uint64_t)(kb * (kAtomBytes >> 4)), sw128_desc(b_addr, 1024), idesc,
                                    kb == 0 ? 1u : 0u);
                     }
-                    if (ok) ptx::mma_commit(&dready[buf]);
+                    if (ok) ptx::mma_commit(&dready[(i & 1) * 2 + buf]);
                 }
                 if (!ok) break;
                 // The item's last copy and its token tile are free once these MMAs complete.
@@ -369,7 +371,12 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             const int nb = min(items[ms].count, kTok);
             for (int nt = 0; nt < g.nnt; ++nt) {
                 const int qn = i * g.nnt + nt, buf = qn & 1;
-                ok = __all_sync(0xFFFFFFFFu, ptx::mbar_wait(&dready[buf], (qn >> 1) & 1, abort, kTimeoutNs));
+                // Earlier N-tiles of this group on buffer buf: per earlier item of the
+                // group, those nt' with the same buffer; in this item, every second nt' < nt.
+                const int m = i >> 1;
+                const int per_item = (g.nnt & 1) ? (g.nnt + (((buf ^ grp) & 1) ? -1 : 1)) / 2 : g.nnt / 2;
+                const uint32_t par = (uint32_t)(m * per_item + (nt >> 1)) & 1u;
+                ok = __all_sync(0xFFFFFFFFu, ptx::mbar_wait(&dready[grp * 2 + buf], par, abort, kTimeoutNs));
                 const int ncols = nt_cols(nt);
                 // Warp eg reads columns [32 eg, 32 eg + 32) of its lanes; lane j < 8 of any
                 // quarter holds token j (D row r is token r % 8).
@@ -465,7 +472,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem_base, g.tmem_cols);
     }
-    if (tid == 0 && *abort) atomicOr(status, STATUS_WAIT_TIMEOUT);
+    if (tid == 0 && *abort) atomicOr(status, STATUS_WAIT_TIMEOUT | STATUS_IN_SCORE);
 }
 
 bool score_tc_shape_supported(int64_t P, int dk) {
