@@ -1,7 +1,7 @@
 """Write a short Markdown summary of ncu output for profiles/.
 
-  launches:  python profiles/summarize_ncu.py launches <launches.csv> <out.md> "<command>"
-  kernel:    python profiles/summarize_ncu.py kernel <report.ncu-rep> <out.md> "<command>" <source.cu> <algorithmic_bytes>
+  launches:  python -m paper_2607_16305_gb300.ncu_summary launches <launches.csv> <out.md> "<command>"
+  kernel:    python -m paper_2607_16305_gb300.ncu_summary kernel <report.ncu-rep> <out.md> "<command>" <source.cu> <algorithmic_bytes>
 
 The kernel summary records DRAM bytes per launch (traffic), throughput, warp
 stall samples and the SHA-256 prefix of the kernel source it was taken on, so
