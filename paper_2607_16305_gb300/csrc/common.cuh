@@ -167,6 +167,11 @@ struct ScoreArgs {
     int32_t* prim_out;
     float* weight_out;
     uint32_t* status;
+    // Optional (tcgen05 level 2): the injection gate decided beside the
+    // bucketing; the value rows of kept tokens are prefetched into L2.
+    const uint8_t* keep_mask;
+    const void* values;   // [S][P][d_v], device memory
+    int64_t vrow_bytes;   // d_v * element size
 };
 cudaError_t launch_score(const LaunchCtx& c, const ScoreArgs& a);
 // Whether the level-2 kernel's shared-memory plan fits this table shape.

@@ -133,7 +133,7 @@ __device__ void block_exclusive_scan3(int3 v, int3& excl, int3& total, int3* war
 }  // namespace
 
 __global__ void __launch_bounds__(kThreads, 1)
-    k2_bucket(unsigned long long* __restrict__ best, int64_t N, int S, int32_t* __restrict__ scene_out,
+    k2_bucket(unsigned long long* best, int64_t N, int S, int32_t* __restrict__ scene_out,
               int32_t* __restrict__ perm, WorkItem* __restrict__ work, int32_t* __restrict__ routed,
               int32_t* __restrict__ counters, const __grid_constant__ GateSpec gate, int smem_bytes) {
     extern __shared__ int cnt[];  // CTA 0: [S] counts, then running token offsets; gate CTAs: priorities

@@ -16,7 +16,7 @@ namespace lookme {
 // One warp per token: ||q_t||_2 (fp32 accumulation of exact bf16/fp32
 // squares) and reset of the token's argmax key.
 template <typename T>
-__global__ void __launch_bounds__(256) k0_prep(const T* __restrict__ q, int64_t N, int dk,
+__global__ void __launch_bounds__(256) k0_prep(const T* q, int64_t N, int dk,
                                                float* __restrict__ qnorm, float* __restrict__ qnorm_out,
                                                unsigned long long* __restrict__ best) {
     pdl_trigger();
@@ -30,7 +30,7 @@ __global__ void __launch_bounds__(256) k0_prep(const T* __restrict__ q, int64_t 
     const int nvec = dk / EPV;
     for (int v = lane; v < nvec; v += 32) {
         float f[EPV];
-        Vec16<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row) + v), f);
+        Vec16<T>::unpack(reinterpret_cast<const uint4*>(row)[v], f);
 #pragma unroll
         for (int i = 0; i < EPV; ++i) acc = fmaf(f[i], f[i], acc);
     }
@@ -65,11 +65,11 @@ __device__ __forceinline__ float level1_score(float dot, float inv_cnorm_s, cons
 // ------------------------------------------------------- K1 on CUDA cores
 // 64 x 64 output tile per CTA, 4 x 4 per thread, k-steps of 16.
 template <typename T>
-__global__ void __launch_bounds__(256) k1_route_simt(const T* __restrict__ q, const T* __restrict__ cent,
+__global__ void __launch_bounds__(256) k1_route_simt(const T* q, const T* __restrict__ cent,
                                                      int64_t N, int64_t S, int dk,
                                                      const float* __restrict__ inv_cnorm,
                                                      const float* __restrict__ bias,
-                                                     const float* __restrict__ qnorm,
+                                                     const float* qnorm,
                                                      unsigned long long* __restrict__ best) {
     __shared__ float As[16][64 + 4];
     __shared__ float Bs[16][64 + 4];

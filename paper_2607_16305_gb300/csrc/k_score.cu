@@ -145,8 +145,8 @@ __device__ __forceinline__ void score_stage(const uint8_t* krow, const float* qf
 
 template <typename T>
 __global__ void __launch_bounds__(k3::kThreads, 1)
-    k3_score(const T* __restrict__ q, const T* __restrict__ keys, int64_t P, int dk, int top_k, float scale,
-             const WorkItem* __restrict__ work, int32_t* __restrict__ counters, const int32_t* __restrict__ perm,
+    k3_score(const T* q, const T* __restrict__ keys, int64_t P, int dk, int top_k, float scale,
+             const WorkItem* work, int32_t* counters, const int32_t* perm,
              int use_slots, int32_t* __restrict__ prim_out, float* __restrict__ weight_out,
              uint32_t* __restrict__ status, const __grid_constant__ k3::Geometry g) {
     using namespace k3;

@@ -115,7 +115,7 @@ inline Geometry geometry(int64_t P, int dk) {
     g.off_z = g.off_b + kBSlots * g.b_bytes;
     g.off_bar = g.off_z + 2 * g.zbytes;
     g.off_meta = g.off_bar + (2 * kMaxStages + 2 * kBSlots + 2 * kISlots + 4 + 2 + 1) * 8;
-    g.smem = g.off_meta + kISlots * ((int)sizeof(WorkItem) + kTok * 4) + 16 + 1024;
+    g.smem = g.off_meta + kISlots * ((int)sizeof(WorkItem) + kTok * 4 + 4) + 16 + 1024;
     return g;
 }
 
@@ -161,28 +161,35 @@ __device__ __noinline__ void mma_kblock(uint32_t live, uint32_t d, uint64_t ad, 
 // serves the warm-up call (prim_out == nullptr: nothing is written) and the
 // real ones.  The common shape (N_p <= 256, top_k <= 8) has a function of its
 // own, so that the larger variants' registers do not weigh on it.
-__device__ __noinline__ void topk_small(const float* z, int64_t P, int top_k, int lane, int64_t t,
-                                        int32_t* prim_out, float* weight_out) {
-    if (P <= 64) k3::topk_token_pop<2, 8>(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
-    else k3::topk_token_pop<8, 8>(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
+// Each returns the lane's selected primitive (lanes < top_k, first 32), else -1.
+__device__ __noinline__ int topk_small(const float* z, int64_t P, int top_k, int lane, int64_t t,
+                                       int32_t* prim_out, float* weight_out) {
+    if (P <= 64) return k3::topk_token_pop<2, 8>(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
+    return k3::topk_token_pop<8, 8>(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
 }
-__device__ __noinline__ void topk_large(const float* z, int64_t P, int top_k, int lane, int64_t t,
-                                        int32_t* prim_out, float* weight_out) {
-    k3::topk_any(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
+__device__ __noinline__ int topk_large(const float* z, int64_t P, int top_k, int lane, int64_t t,
+                                       int32_t* prim_out, float* weight_out) {
+    return k3::topk_any(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
 }
-__device__ __forceinline__ void topk_item(const float* z, int64_t P, int top_k, int lane, int64_t t,
-                                          int32_t* prim_out, float* weight_out) {
-    if (P <= 256 && top_k <= 8) topk_small(z, P, top_k, lane, t, prim_out, weight_out);
-    else topk_large(z, P, top_k, lane, t, prim_out, weight_out);
+__device__ __forceinline__ int topk_item(const float* z, int64_t P, int top_k, int lane, int64_t t,
+                                         int32_t* prim_out, float* weight_out) {
+    if (P <= 256 && top_k <= 8) return topk_small(z, P, top_k, lane, t, prim_out, weight_out);
+    return topk_large(z, P, top_k, lane, t, prim_out, weight_out);
+}
+
+// Pull one value row into L2 (128-byte lines, no register result).
+__device__ __forceinline__ void prefetch_row_l2(const uint8_t* row, int64_t bytes) {
+    for (int64_t o = 0; o < bytes; o += 128) asm volatile("prefetch.global.L2 [%0];" ::"l"(row + o));
 }
 
 }  // namespace k3tc
 
 __global__ void __launch_bounds__(k3tc::kThreads, 1)
-    k3_score_tc(const uint8_t* __restrict__ keys_t, int64_t block_bytes, const __nv_bfloat16* __restrict__ q,
-                int64_t P, int dk, int top_k, float scale, const WorkItem* __restrict__ work,
-                const int32_t* __restrict__ counters, const int32_t* __restrict__ perm, int use_slots,
+    k3_score_tc(const uint8_t* __restrict__ keys_t, int64_t block_bytes, const __nv_bfloat16* q,
+                int64_t P, int dk, int top_k, float scale, const WorkItem* work,
+                const int32_t* counters, const int32_t* perm, int use_slots,
                 int32_t* __restrict__ prim_out, float* __restrict__ weight_out, uint32_t* __restrict__ status,
+                const uint8_t* keep_mask, const uint8_t* __restrict__ values, int64_t vrow_bytes,
                 const __grid_constant__ k3tc::Geometry g) {
     using namespace k3tc;
     extern __shared__ uint8_t smem_raw[];
@@ -205,7 +212,8 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
     uint64_t* drain = tempty + 2;
     WorkItem* items = reinterpret_cast<WorkItem*>(smem + g.off_meta);
     int32_t* toks = reinterpret_cast<int32_t*>(items + kISlots);
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(toks + kISlots * kTok);
+    uint32_t* keepbits = reinterpret_cast<uint32_t*>(toks + kISlots * kTok);  // gate of the item's tokens
+    uint32_t* tmem_slot = keepbits + kISlots;
     volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int tid = threadIdx.x, lane = tid % 32, warp = tid / 32;
@@ -216,22 +224,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
     } else if (warp >= 2 && warp < kBuildWarp) {
         topk_item(zs, P, top_k, lane, 0, nullptr, nullptr);
     }
-    // The work list is the predecessor's output; TMEM is allocated only after
-    // this wait, so a CTA that holds TMEM never waits on an earlier kernel.
-    pdl_wait();
-    const int n_work = counters[0];
-    const int G = gridDim.x;
-    const int my_items = n_work > (int)blockIdx.x ? (n_work - (int)blockIdx.x + G - 1) / G : 0;
-    if (my_items == 0) return;  // uniform for the CTA: nothing allocated yet
-    auto item_index = [&](int i) { return (int)blockIdx.x + i * G; };
-    // N-tile nt: its first sub-block, its sub-block count (1 or 2) and its N.
-    auto nt_base = [&](int nt) { return nt * 2 * g.nkb; };
-    auto nt_subs = [&](int nt) { return (nt == g.nnt - 1 && (g.ntile & 1)) ? 1 : 2; };
-    auto nt_cols = [&](int nt) {
-        const int64_t rows = P - (int64_t)nt * kNTile;
-        return (int)(rows >= kNTile ? kNTile : (rows + 15) / 16 * 16);
-    };
-
+    // Barriers are initialised before the dependency wait (shared memory only).
     if (tid == 0) {
         for (int i = 0; i < g.n_stages; ++i) {
             ptx::mbar_init(&full[i], 1);
@@ -251,11 +244,34 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         *abort = 0;
         ptx::fence_mbar_init();
     }
-    if (warp == 1) ptx::tmem_alloc(tmem_slot, g.tmem_cols);
-    ptx::tc_fence_before();
     __syncthreads();
-    ptx::tc_fence_after();
-    const uint32_t tmem_base = *tmem_slot;
+    // The work list is the predecessor's output (read with plain loads: no
+    // read-only/restrict qualifier lets the compiler move them above the
+    // wait); TMEM is allocated only after it, so a CTA that holds TMEM never
+    // waits on an earlier kernel.
+    pdl_wait();
+    const int n_work = counters[0];
+    const int G = gridDim.x;
+    const int my_items = n_work > (int)blockIdx.x ? (n_work - (int)blockIdx.x + G - 1) / G : 0;
+    if (my_items == 0) return;  // uniform for the CTA: nothing allocated yet
+    auto item_index = [&](int i) { return (int)blockIdx.x + i * G; };
+    // N-tile nt: its first sub-block, its sub-block count (1 or 2) and its N.
+    auto nt_base = [&](int nt) { return nt * 2 * g.nkb; };
+    auto nt_subs = [&](int nt) { return (nt == g.nnt - 1 && (g.ntile & 1)) ? 1 : 2; };
+    auto nt_cols = [&](int nt) {
+        const int64_t rows = P - (int64_t)nt * kNTile;
+        return (int)(rows >= kNTile ? kNTile : (rows + 15) / 16 * 16);
+    };
+    // The producer starts the key stream at once; the other warps meet on
+    // named barrier 4 for the TMEM address.
+    uint32_t tmem_base = 0;
+    if (warp != 0) {
+        if (warp == 1) ptx::tmem_alloc(tmem_slot, g.tmem_cols);
+        ptx::tc_fence_before();
+        asm volatile("bar.sync 4, %0;" ::"n"(kThreads - 32) : "memory");
+        ptx::tc_fence_after();
+        tmem_base = *tmem_slot;
+    }
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer
@@ -403,7 +419,12 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
                 if (lane == 0) ptx::mbar_arrive(&tempty[buf]);
             }
             if (k3tc::group_sync_or(grp, *abort)) break;  // all logits of the item are in shared memory
-            if (eg < nb) k3tc::topk_item(zg + eg, P, top_k, lane, toks[ms * kTok + eg], prim_out, weight_out);
+            if (eg < nb) {
+                const int pj = k3tc::topk_item(zg + eg, P, top_k, lane, toks[ms * kTok + eg], prim_out, weight_out);
+                // A kept token's value rows are read by the injection next: start them now.
+                if (keep_mask && pj >= 0 && ((keepbits[ms] >> eg) & 1u))
+                    k3tc::prefetch_row_l2(values + ((int64_t)items[ms].scene * P + pj) * vrow_bytes, vrow_bytes);
+            }
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&iempty[ms]);
         }
@@ -416,6 +437,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         const uint4* qv = reinterpret_cast<const uint4*>(q);
         WorkItem w = work[item_index(0)];
         int32_t tok = lane < w.count ? perm[w.begin + lane] : 0;
+        bool kp = keep_mask && lane < w.count && keep_mask[tok];
         bool ok = true;
         for (int i = 0; i < my_items; ++i) {
             const int ms = i % kISlots, bs = i % kBSlots;
@@ -428,6 +450,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             uint8_t* bt = btile + bs * g.b_bytes;
             WorkItem wn = w;
             int32_t tokn = 0;
+            bool kpn = false;
             for (int base = 0; base < total; base += 32 * kQBatch) {
                 uint4 v[kQBatch];
                 int jj[kQBatch], cc[kQBatch];
@@ -455,7 +478,12 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             if (i + 1 < my_items) tokn = lane < wn.count ? perm[wn.begin + lane] : 0;
             ptx::fence_proxy_async_smem();  // the tile is read by the tensor core (async proxy)
             if (lane < nb) toks[ms * kTok + lane] = tok;
-            if (lane == 0) items[ms] = w;
+            const uint32_t kb = __ballot_sync(0xFFFFFFFFu, kp);
+            if (lane == 0) {
+                items[ms] = w;
+                keepbits[ms] = kb;
+            }
+            if (i + 1 < my_items) kpn = keep_mask && lane < wn.count && keep_mask[tokn];
             __syncwarp();
             if (lane == 0) {
                 ptx::mbar_arrive(&ifull[ms]);
@@ -463,6 +491,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             }
             w = wn;
             tok = tokn;
+            kp = kpn;
         }
     }
 
@@ -492,7 +521,7 @@ cudaError_t launch_score_tc(const LaunchCtx& c, const void* keys_tiled, const Sc
     return launch_pdl(k3_score_tc, dim3(c.num_sms), dim3(k3tc::kThreads), (size_t)g.smem, c.stream,
                       (const uint8_t*)keys_tiled, (int64_t)g.spi * k3tc::kSubBytes, (const __nv_bfloat16*)a.q, a.P,
                       a.dk, a.top_k, a.scale, a.work, (const int32_t*)a.counters, a.perm, a.use_slots, a.prim_out,
-                      a.weight_out, a.status, g);
+                      a.weight_out, a.status, a.keep_mask, (const uint8_t*)a.values, a.vrow_bytes, g);
 }
 
 cudaError_t configure_score_tc_kernel() {

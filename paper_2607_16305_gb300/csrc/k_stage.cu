@@ -16,8 +16,7 @@ namespace lookme {
 
 __global__ void __launch_bounds__(256) k6_stage(const uint4* __restrict__ keys_host, uint4* __restrict__ slots,
                                                 int64_t block_vecs, int64_t n_slots,
-                                                const int32_t* __restrict__ routed,
-                                                const int32_t* __restrict__ counters) {
+                                                const int32_t* routed, const int32_t* counters) {
     pdl_trigger();
     pdl_wait();
     const int64_t n_routed = min((int64_t)counters[1], n_slots);

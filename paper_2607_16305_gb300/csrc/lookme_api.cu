@@ -563,6 +563,11 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
     a.prim_out = prim_out;
     a.weight_out = weight_out;
     a.status = t->status;
+    // With the gate decided beside the bucketing, level 2 prefetches the kept
+    // tokens' value rows (HBM-resident tables).
+    a.keep_mask = (gate && d.residency == LOOKME_RES_DEVICE) ? gate->mask : nullptr;
+    a.values = t->values;
+    a.vrow_bytes = d.d_value * (int64_t)t->esz;
     st = launch(t, s, KID_SCORE,
                 [&] { return t->tc_score ? launch_score_tc(ctx, a.keys, a) : launch_score(ctx, a); });
     if (st != LOOKME_OK) return st;

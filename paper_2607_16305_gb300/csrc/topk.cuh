@@ -17,7 +17,7 @@ __device__ __forceinline__ float from_orderable(uint32_t u) {
 // index on ties) and the
 // softmax over the selected logits; writes prim/weight of token t (nothing
 // when prim_out is null).
-__device__ __forceinline__ void topk_token(const float* z, int64_t P, int top_k, int lane, int64_t t,
+__device__ __forceinline__ int topk_token(const float* z, int64_t P, int top_k, int lane, int64_t t,
                                            int32_t* prim_out, float* weight_out, int zs = 1) {
     // Each lane keeps the best untaken element of its slice p = lane + 32 i.
     uint64_t taken = 0ull;
@@ -74,12 +74,13 @@ __device__ __forceinline__ void topk_token(const float* z, int64_t P, int top_k,
             weight_out[t * top_k + j] = e[h] / sum;
         }
     }
+    return lane < top_k ? my_p[0] : -1;
 }
 // Register-resident variant for N_p <= 32 * PPL: each lane holds the order
 // keys of its elements p = 32 i + lane, so a round is an unrolled scan of
 // PPL registers plus two warp reductions.  Same result as topk_token.
 template <int PPL>
-__device__ __forceinline__ void topk_token_regs(const float* z, int64_t P, int top_k, int lane, int64_t t,
+__device__ __forceinline__ int topk_token_regs(const float* z, int64_t P, int top_k, int lane, int64_t t,
                                                 int32_t* prim_out, float* weight_out, int zs = 1) {
     uint32_t key[PPL];
 #pragma unroll
@@ -133,6 +134,7 @@ __device__ __forceinline__ void topk_token_regs(const float* z, int64_t P, int t
             weight_out[t * top_k + j] = e[h] / sum;
         }
     }
+    return lane < top_k ? my_p[0] : -1;
 }
 
 // Sorted-list variant for top_k <= L (L = 8 or 16), N_p <= 32 * PPL.  An
@@ -186,7 +188,7 @@ __device__ __forceinline__ void merge_top_desc(uint64_t (&a)[L], const uint64_t 
 }
 
 template <int PPL, int L>
-__device__ __forceinline__ void topk_token_pop(const float* z, int64_t P, int top_k, int lane, int64_t t,
+__device__ __forceinline__ int topk_token_pop(const float* z, int64_t P, int top_k, int lane, int64_t t,
                                                int32_t* prim_out, float* weight_out, int zs = 1) {
     constexpr int G = (PPL + L - 1) / L;  // groups of L elements per lane
     uint64_t a[L];
@@ -235,31 +237,30 @@ __device__ __forceinline__ void topk_token_pop(const float* z, int64_t P, int to
         prim_out[t * top_k + lane] = (int32_t)my_p;
         weight_out[t * top_k + lane] = e / sum;
     }
+    return lane < top_k ? (int)my_p : -1;
 }
 
 // Top-k of one token, picking the register-resident variant when N_p allows.
-__device__ __forceinline__ void topk_any(const float* z, int64_t P, int top_k, int lane, int64_t t,
+__device__ __forceinline__ int topk_any(const float* z, int64_t P, int top_k, int lane, int64_t t,
                                          int32_t* prim_out, float* weight_out, int zs = 1) {
     if (top_k <= 8) {
-        if (P <= 64) topk_token_pop<2, 8>(z, P, top_k, lane, t, prim_out, weight_out, zs);
-        else if (P <= 256) topk_token_pop<8, 8>(z, P, top_k, lane, t, prim_out, weight_out, zs);
-        else if (P <= 512) topk_token_pop<16, 8>(z, P, top_k, lane, t, prim_out, weight_out, zs);
-        else if (P <= 1024) topk_token_pop<32, 8>(z, P, top_k, lane, t, prim_out, weight_out, zs);
-        else topk_token(z, P, top_k, lane, t, prim_out, weight_out, zs);
-        return;
+        if (P <= 64) return topk_token_pop<2, 8>(z, P, top_k, lane, t, prim_out, weight_out, zs);
+        else if (P <= 256) return topk_token_pop<8, 8>(z, P, top_k, lane, t, prim_out, weight_out, zs);
+        else if (P <= 512) return topk_token_pop<16, 8>(z, P, top_k, lane, t, prim_out, weight_out, zs);
+        else if (P <= 1024) return topk_token_pop<32, 8>(z, P, top_k, lane, t, prim_out, weight_out, zs);
+        return topk_token(z, P, top_k, lane, t, prim_out, weight_out, zs);
     }
     if (top_k <= 16 && P <= 1024) {
-        if (P <= 512) topk_token_pop<16, 16>(z, P, top_k, lane, t, prim_out, weight_out, zs);
-        else topk_token_pop<32, 16>(z, P, top_k, lane, t, prim_out, weight_out, zs);
-        return;
+        if (P <= 512) return topk_token_pop<16, 16>(z, P, top_k, lane, t, prim_out, weight_out, zs);
+        return topk_token_pop<32, 16>(z, P, top_k, lane, t, prim_out, weight_out, zs);
     }
-    if (P <= 32) topk_token_regs<1>(z, P, top_k, lane, t, prim_out, weight_out, zs);
-    else if (P <= 64) topk_token_regs<2>(z, P, top_k, lane, t, prim_out, weight_out, zs);
-    else if (P <= 128) topk_token_regs<4>(z, P, top_k, lane, t, prim_out, weight_out, zs);
-    else if (P <= 256) topk_token_regs<8>(z, P, top_k, lane, t, prim_out, weight_out, zs);
-    else if (P <= 512) topk_token_regs<16>(z, P, top_k, lane, t, prim_out, weight_out, zs);
-    else if (P <= 1024) topk_token_regs<32>(z, P, top_k, lane, t, prim_out, weight_out, zs);
-    else topk_token(z, P, top_k, lane, t, prim_out, weight_out, zs);
+    if (P <= 32) return topk_token_regs<1>(z, P, top_k, lane, t, prim_out, weight_out, zs);
+    if (P <= 64) return topk_token_regs<2>(z, P, top_k, lane, t, prim_out, weight_out, zs);
+    if (P <= 128) return topk_token_regs<4>(z, P, top_k, lane, t, prim_out, weight_out, zs);
+    if (P <= 256) return topk_token_regs<8>(z, P, top_k, lane, t, prim_out, weight_out, zs);
+    if (P <= 512) return topk_token_regs<16>(z, P, top_k, lane, t, prim_out, weight_out, zs);
+    if (P <= 1024) return topk_token_regs<32>(z, P, top_k, lane, t, prim_out, weight_out, zs);
+    return topk_token(z, P, top_k, lane, t, prim_out, weight_out, zs);
 }
 
 }  // namespace k3
