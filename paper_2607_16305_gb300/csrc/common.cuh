@@ -161,6 +161,7 @@ struct ScoreArgs {
     int top_k;
     float scale;          // 1 / sqrt(d_k)
     const WorkItem* work;
+    int64_t work_cap;     // entries of the work array
     int32_t* counters;    // [0] work items (from bucketing), [3] work-taking counter (reset by bucketing)
     const int32_t* perm;
     int use_slots;        // index key blocks by WorkItem::slot instead of ::scene

@@ -114,7 +114,7 @@ inline Geometry geometry(int64_t P, int dk) {
     g.off_b = g.n_stages * g.slot_bytes;
     g.off_z = g.off_b + kBSlots * g.b_bytes;
     g.off_bar = g.off_z + 2 * g.zbytes;
-    g.off_meta = g.off_bar + (2 * kMaxStages + 2 * kBSlots + 2 * kISlots + 4 + 2 + 1) * 8;
+    g.off_meta = g.off_bar + (2 * kMaxStages + 2 * kBSlots + 2 * kISlots + 4 + 2 + 1 + 2) * 8;
     g.smem = g.off_meta + kISlots * ((int)sizeof(WorkItem) + kTok * 4 + 4) + 16 + 1024;
     return g;
 }
@@ -187,7 +187,7 @@ __device__ __forceinline__ void prefetch_row_l2(const uint8_t* row, int64_t byte
 __global__ void __launch_bounds__(k3tc::kThreads, 1)
     k3_score_tc(const uint8_t* __restrict__ keys_t, int64_t block_bytes, const __nv_bfloat16* q,
                 int64_t P, int dk, int top_k, float scale, const WorkItem* work,
-                const int32_t* counters, const int32_t* perm, int use_slots,
+                const int32_t* counters, const int32_t* perm, int64_t work_cap, int use_slots,
                 int32_t* __restrict__ prim_out, float* __restrict__ weight_out, uint32_t* __restrict__ status,
                 const uint8_t* keep_mask, const uint8_t* __restrict__ values, int64_t vrow_bytes,
                 const __grid_constant__ k3tc::Geometry g) {
@@ -210,6 +210,8 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
     uint64_t* dready = iempty + kISlots;
     uint64_t* tempty = dready + 4;
     uint64_t* drain = tempty + 2;
+    uint64_t* setup = drain + 1;      // the other barriers are initialised (thread 0)
+    uint64_t* tmem_ready = setup + 1; // the TMEM address is in tmem_slot (warp 1)
     WorkItem* items = reinterpret_cast<WorkItem*>(smem + g.off_meta);
     int32_t* toks = reinterpret_cast<int32_t*>(items + kISlots);
     uint32_t* keepbits = reinterpret_cast<uint32_t*>(toks + kISlots * kTok);  // gate of the item's tokens
@@ -218,13 +220,35 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
 
     const int tid = threadIdx.x, lane = tid % 32, warp = tid / 32;
     pdl_trigger();
+    // Two hand-off barriers first, so that after the dependency wait no role
+    // waits for another role's warm-up: only for what it actually needs.
+    if (tid == 0) {
+        ptx::mbar_init(setup, 1);
+        ptx::mbar_init(tmem_ready, 1);
+        *abort = 0;
+        ptx::fence_mbar_init();
+    }
+    __syncthreads();
     // Warm-up while the predecessor finishes: no memory, barrier or TMEM effect.
     if (warp == 1 && lane == 0) {
         mma_kblock(0u, 0u, 0ull, 0ull, idesc_m128(kNTile), 1u);
     } else if (warp >= 2 && warp < kBuildWarp) {
         topk_item(zs, P, top_k, lane, 0, nullptr, nullptr);
     }
-    // Barriers are initialised before the dependency wait (shared memory only).
+    // The work list is the predecessor's output (read with plain loads: a
+    // read-only/restrict qualifier would let the compiler move them above the
+    // wait); TMEM is allocated only after it, so a CTA that holds TMEM never
+    // waits on an earlier kernel.
+    pdl_wait();
+    // This CTA's first work entry is read together with the count (the work
+    // array holds work_cap entries), saving a dependent round trip.
+    WorkItem w0;
+    w0.scene = w0.begin = w0.count = w0.slot = 0;
+    if ((int64_t)blockIdx.x < work_cap) w0 = work[blockIdx.x];
+    const int n_work = counters[0];
+    const int G = gridDim.x;
+    const int my_items = n_work > (int)blockIdx.x ? (n_work - (int)blockIdx.x + G - 1) / G : 0;
+    if (my_items == 0) return;  // uniform for the CTA: nothing allocated yet
     if (tid == 0) {
         for (int i = 0; i < g.n_stages; ++i) {
             ptx::mbar_init(&full[i], 1);
@@ -241,19 +265,9 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         for (int i = 0; i < 4; ++i) ptx::mbar_init(&dready[i], 1);
         for (int i = 0; i < 2; ++i) ptx::mbar_init(&tempty[i], kGroupWarps);
         ptx::mbar_init(drain, 1);
-        *abort = 0;
         ptx::fence_mbar_init();
+        ptx::mbar_arrive(setup);
     }
-    __syncthreads();
-    // The work list is the predecessor's output (read with plain loads: no
-    // read-only/restrict qualifier lets the compiler move them above the
-    // wait); TMEM is allocated only after it, so a CTA that holds TMEM never
-    // waits on an earlier kernel.
-    pdl_wait();
-    const int n_work = counters[0];
-    const int G = gridDim.x;
-    const int my_items = n_work > (int)blockIdx.x ? (n_work - (int)blockIdx.x + G - 1) / G : 0;
-    if (my_items == 0) return;  // uniform for the CTA: nothing allocated yet
     auto item_index = [&](int i) { return (int)blockIdx.x + i * G; };
     // N-tile nt: its first sub-block, its sub-block count (1 or 2) and its N.
     auto nt_base = [&](int nt) { return nt * 2 * g.nkb; };
@@ -262,13 +276,19 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         const int64_t rows = P - (int64_t)nt * kNTile;
         return (int)(rows >= kNTile ? kNTile : (rows + 15) / 16 * 16);
     };
-    // The producer starts the key stream at once; the other warps meet on
-    // named barrier 4 for the TMEM address.
+    // The producer (thread 0 initialised the barriers) starts the key stream
+    // at once; the others wait for the barriers, and the MMA issuer and the
+    // epilogue for the TMEM address, which warp 1 publishes.
     uint32_t tmem_base = 0;
-    if (warp != 0) {
-        if (warp == 1) ptx::tmem_alloc(tmem_slot, g.tmem_cols);
+    if (warp != 0 && warp != kBuildWarp) ptx::mbar_wait(setup, 0, abort, kTimeoutNs);
+    if (warp == 1) {
+        ptx::tmem_alloc(tmem_slot, g.tmem_cols);
         ptx::tc_fence_before();
-        asm volatile("bar.sync 4, %0;" ::"n"(kThreads - 32) : "memory");
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(tmem_ready);
+    }
+    if (warp >= 1 && warp < kBuildWarp) {
+        ptx::mbar_wait(tmem_ready, 0, abort, kTimeoutNs);
         ptx::tc_fence_after();
         tmem_base = *tmem_slot;
     }
@@ -304,7 +324,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             }
         };
         // The work entry of the next item is loaded while this one's copies go out.
-        WorkItem w = work[item_index(0)];
+        WorkItem w = w0;
         for (int i = 0; i < my_items && ok; ++i) {
             WorkItem wn = w;
             if (i + 1 < my_items) wn = work[item_index(i + 1)];
@@ -435,13 +455,16 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             reinterpret_cast<uint4*>(btile)[idx] = make_uint4(0u, 0u, 0u, 0u);
         const int cpr = g.row_bytes / 16;  // 16-byte chunks per query row
         const uint4* qv = reinterpret_cast<const uint4*>(q);
-        WorkItem w = work[item_index(0)];
+        WorkItem w = w0;
         int32_t tok = lane < w.count ? perm[w.begin + lane] : 0;
         bool kp = keep_mask && lane < w.count && keep_mask[tok];
         bool ok = true;
         for (int i = 0; i < my_items; ++i) {
             const int ms = i % kISlots, bs = i % kBSlots;
-            if (lane == 0)
+            // The first item's slots are free by construction: its query rows are
+            // loaded before this warp touches any barrier (and before the key
+            // stream fills the memory system).
+            if (lane == 0 && i > 0)
                 ok = ptx::mbar_wait(&iempty[ms], ((i / kISlots) & 1) ^ 1, abort, kTimeoutNs) &&
                      ptx::mbar_wait(&bempty[bs], ((i / kBSlots) & 1) ^ 1, abort, kTimeoutNs);
             if (!__shfl_sync(0xFFFFFFFFu, (int)ok, 0)) break;
@@ -476,6 +499,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             }
             if (total == 0 && i + 1 < my_items) wn = work[item_index(i + 1)];
             if (i + 1 < my_items) tokn = lane < wn.count ? perm[wn.begin + lane] : 0;
+            if (i == 0 && !__all_sync(0xFFFFFFFFu, ptx::mbar_wait(setup, 0, abort, kTimeoutNs))) break;
             ptx::fence_proxy_async_smem();  // the tile is read by the tensor core (async proxy)
             if (lane < nb) toks[ms * kTok + lane] = tok;
             const uint32_t kb = __ballot_sync(0xFFFFFFFFu, kp);
@@ -520,7 +544,7 @@ cudaError_t launch_score_tc(const LaunchCtx& c, const void* keys_tiled, const Sc
     if (!score_tc_shape_supported(a.P, a.dk)) return cudaErrorInvalidConfiguration;
     return launch_pdl(k3_score_tc, dim3(c.num_sms), dim3(k3tc::kThreads), (size_t)g.smem, c.stream,
                       (const uint8_t*)keys_tiled, (int64_t)g.spi * k3tc::kSubBytes, (const __nv_bfloat16*)a.q, a.P,
-                      a.dk, a.top_k, a.scale, a.work, (const int32_t*)a.counters, a.perm, a.use_slots, a.prim_out,
+                      a.dk, a.top_k, a.scale, a.work, (const int32_t*)a.counters, a.perm, a.work_cap, a.use_slots, a.prim_out,
                       a.weight_out, a.status, a.keep_mask, (const uint8_t*)a.values, a.vrow_bytes, g);
 }
 

@@ -557,6 +557,7 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
     a.top_k = top_k;
     a.scale = (float)(1.0 / std::sqrt((double)dk));
     a.work = t->work;
+    a.work_cap = t->cap + d.n_scenes;
     a.counters = t->counters;
     a.perm = t->perm;
     a.use_slots = staged ? 1 : 0;
