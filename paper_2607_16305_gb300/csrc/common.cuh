@@ -91,9 +91,9 @@ __device__ __forceinline__ int32_t unpack_scene(unsigned long long key, int64_t 
     return (key == 0ull || s >= (uint64_t)n_scenes) ? 0 : (int32_t)s;
 }
 
-// Work item of level 2: tokens perm[begin, begin + count) all routed to
-// `scene`; `slot` is the scene's index in the routed-scene list (and its HBM
-// slot when keys are staged).
+// Work item i of level 2: tokens item_tok[begin, begin + count) all routed to
+// `scene`, begin = kTokensPerItem * i; `slot` is the scene's index in the
+// routed-scene list (and its HBM slot when keys are staged).
 struct WorkItem {
     int32_t scene, begin, count, slot;
 };
@@ -149,7 +149,7 @@ constexpr int kTokensPerItem = 8;
 // gate (optional, GateSpec declared below) adds CTAs that compute the injection gate.
 struct GateSpec;
 cudaError_t launch_bucket(const LaunchCtx& c, unsigned long long* best, int64_t N, int64_t S,
-                          int32_t* scene_out, int32_t* perm, WorkItem* work, int32_t* routed, int32_t* counters,
+                          int32_t* scene_out, int32_t* item_tok, WorkItem* work, int32_t* routed, int32_t* counters,
                           const GateSpec* gate = nullptr);
 // K3
 struct ScoreArgs {
@@ -163,7 +163,7 @@ struct ScoreArgs {
     const WorkItem* work;
     int64_t work_cap;     // entries of the work array
     int32_t* counters;    // [0] work items (from bucketing), [3] work-taking counter (reset by bucketing)
-    const int32_t* perm;
+    const int32_t* item_tok;  // the items' token ids, kTokensPerItem slots per work entry
     int use_slots;        // index key blocks by WorkItem::slot instead of ::scene
     int32_t* prim_out;
     float* weight_out;

@@ -4,10 +4,12 @@
 //
 // Outputs
 //   scene_out[t]   the routed scene of every token (decoded argmax key)
-//   perm           token ids grouped by scene (scene-major; order inside a
-//                  scene is unspecified)
 //   work           level-2 work items (scene, begin, count <= 8, slot) in
 //                  scene order: every scene's bucket cut into chunks
+//   item_tok       the items' token ids, item-major: item i's tokens at
+//                  [8 i, 8 i + count) (begin = 8 i), so a consumer that knows
+//                  an item's index reads its tokens without first reading the
+//                  item; order inside a scene is unspecified
 //   routed         the distinct routed scenes in increasing order; a scene's
 //                  position in it is its `slot`
 //   counters[0..3] number of work items, of routed scenes, largest bucket;
@@ -91,53 +93,49 @@ __device__ void gate_block(const GateSpec& gs, float* buf, int cap) {
         if (keep) gs.sel[gs.sel_base[sg] + rank] = (int32_t)t;
     }
 }
-// Exclusive block-wide scan of three counters at once.
-__device__ void block_exclusive_scan3(int3 v, int3& excl, int3& total, int3* warp_buf) {
+// Exclusive block-wide scan of two counters at once.
+__device__ void block_exclusive_scan2(int2 v, int2& excl, int2& total, int2* warp_buf) {
     const int lane = threadIdx.x % 32, warp = threadIdx.x / 32;
-    int3 inc = v;
+    int2 inc = v;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
         const int a = __shfl_up_sync(0xFFFFFFFFu, inc.x, o);
         const int b = __shfl_up_sync(0xFFFFFFFFu, inc.y, o);
-        const int c = __shfl_up_sync(0xFFFFFFFFu, inc.z, o);
         if (lane >= o) {
             inc.x += a;
             inc.y += b;
-            inc.z += c;
         }
     }
     if (lane == 31) warp_buf[warp] = inc;
     __syncthreads();
     if (warp == 0) {
-        int3 w = lane < kThreads / 32 ? warp_buf[lane] : make_int3(0, 0, 0);
-        int3 wi = w;
+        int2 w = lane < kThreads / 32 ? warp_buf[lane] : make_int2(0, 0);
+        int2 wi = w;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int a = __shfl_up_sync(0xFFFFFFFFu, wi.x, o);
             const int b = __shfl_up_sync(0xFFFFFFFFu, wi.y, o);
-            const int c = __shfl_up_sync(0xFFFFFFFFu, wi.z, o);
             if (lane >= o) {
                 wi.x += a;
                 wi.y += b;
-                wi.z += c;
             }
         }
-        if (lane < kThreads / 32) warp_buf[lane] = make_int3(wi.x - w.x, wi.y - w.y, wi.z - w.z);
+        if (lane < kThreads / 32) warp_buf[lane] = make_int2(wi.x - w.x, wi.y - w.y);
         if (lane == kThreads / 32 - 1) warp_buf[32] = wi;
     }
     __syncthreads();
-    const int3 wb = warp_buf[warp];
-    excl = make_int3(wb.x + inc.x - v.x, wb.y + inc.y - v.y, wb.z + inc.z - v.z);
+    const int2 wb = warp_buf[warp];
+    excl = make_int2(wb.x + inc.x - v.x, wb.y + inc.y - v.y);
     total = warp_buf[32];
 }
 }  // namespace
 
 __global__ void __launch_bounds__(kThreads, 1)
     k2_bucket(unsigned long long* best, int64_t N, int S, int32_t* __restrict__ scene_out,
-              int32_t* __restrict__ perm, WorkItem* __restrict__ work, int32_t* __restrict__ routed,
+              int32_t* __restrict__ item_tok, WorkItem* __restrict__ work, int32_t* __restrict__ routed,
               int32_t* __restrict__ counters, const __grid_constant__ GateSpec gate, int smem_bytes) {
-    extern __shared__ int cnt[];  // CTA 0: [S] counts, then running token offsets; gate CTAs: priorities
-    __shared__ int3 warp_buf[33];
+    extern __shared__ int cnt[];  // CTA 0: [S] counts, then running item_tok positions; gate CTAs: priorities
+    __shared__ int2 warp_buf[33];
     __shared__ int max_bucket;
     pdl_trigger();
     pdl_wait();
@@ -159,54 +157,53 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Each thread owns a contiguous run of scenes.
     const int per = (S + kThreads - 1) / kThreads;
     const int s0 = min(S, tid * per), s1 = min(S, s0 + per);
-    int3 mine = make_int3(0, 0, 0);  // tokens, work items, routed scenes
+    int2 mine = make_int2(0, 0);  // work items, routed scenes
     int mx = 0;
     for (int s = s0; s < s1; ++s) {
         const int c = cnt[s];
-        mine.x += c;
-        mine.y += (c + kTokensPerItem - 1) / kTokensPerItem;
-        mine.z += c > 0;
+        mine.x += (c + kTokensPerItem - 1) / kTokensPerItem;
+        mine.y += c > 0;
         mx = max(mx, c);
     }
-    int3 base, total;
-    block_exclusive_scan3(mine, base, total, warp_buf);
+    int2 base, total;
+    block_exclusive_scan2(mine, base, total, warp_buf);
     if (mx) atomicMax(&max_bucket, mx);
 
-    int tok = base.x, wi = base.y, slot = base.z;
+    int wi = base.x, slot = base.y;
     for (int s = s0; s < s1; ++s) {
         const int c = cnt[s];
-        cnt[s] = tok;
+        cnt[s] = wi * kTokensPerItem;  // the scene's first item_tok position
         if (c > 0) {
             routed[slot] = s;
             for (int b = 0; b < c; b += kTokensPerItem) {
                 WorkItem w;
                 w.scene = s;
-                w.begin = tok + b;
+                w.begin = wi * kTokensPerItem;
                 w.count = min(kTokensPerItem, c - b);
                 w.slot = slot;
                 work[wi++] = w;
             }
             ++slot;
         }
-        tok += c;
     }
     __syncthreads();
     if (tid == 0) {
-        counters[0] = total.y;
-        counters[1] = total.z;
+        counters[0] = total.x;
+        counters[1] = total.y;
         counters[2] = max_bucket;
         counters[3] = 0;  // level-2 work-taking counter
     }
     for (int64_t t = tid; t < N; t += kThreads) {
         const int32_t s = unpack_scene(best[t], S);
         best[t] = 0ull;  // ready for the next call's argmax
+        // A scene's k-th token lands in its item k / 8, lane k % 8.
         const int pos = atomicAdd(&cnt[s], 1);
-        perm[pos] = (int32_t)t;
+        item_tok[pos] = (int32_t)t;
     }
 }
 
 cudaError_t launch_bucket(const LaunchCtx& c, unsigned long long* best, int64_t N, int64_t S,
-                          int32_t* scene_out, int32_t* perm, WorkItem* work, int32_t* routed, int32_t* counters,
+                          int32_t* scene_out, int32_t* item_tok, WorkItem* work, int32_t* routed, int32_t* counters,
                           const GateSpec* gate) {
     GateSpec gs;
     if (gate) {
@@ -217,7 +214,7 @@ cudaError_t launch_bucket(const LaunchCtx& c, unsigned long long* best, int64_t 
     const int gate_ctas = gate ? (int)((N + kGateTokens - 1) / kGateTokens) : 0;
     const int smem = (int)std::max<int64_t>(S * (int64_t)sizeof(int), gate ? kGateStage : 0);
     return launch_pdl(k2_bucket, dim3(1 + gate_ctas), dim3(kThreads), (size_t)smem, c.stream, best, N, (int)S,
-                      scene_out, perm, work, routed, counters, gs, smem);
+                      scene_out, item_tok, work, routed, counters, gs, smem);
 }
 
 cudaError_t configure_bucket_kernel() {

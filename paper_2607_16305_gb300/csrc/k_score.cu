@@ -146,7 +146,7 @@ __device__ __forceinline__ void score_stage(const uint8_t* krow, const float* qf
 template <typename T>
 __global__ void __launch_bounds__(k3::kThreads, 1)
     k3_score(const T* q, const T* __restrict__ keys, int64_t P, int dk, int top_k, float scale,
-             const WorkItem* work, int32_t* counters, const int32_t* perm,
+             const WorkItem* work, int32_t* counters, const int32_t* item_tok,
              int use_slots, int32_t* __restrict__ prim_out, float* __restrict__ weight_out,
              uint32_t* __restrict__ status, const __grid_constant__ k3::Geometry g) {
     using namespace k3;
@@ -214,7 +214,7 @@ __global__ void __launch_bounds__(k3::kThreads, 1)
             const WorkItem w = work[wi];
             int32_t t = 0;
             if (lane < w.count) {
-                t = perm[w.begin + lane];
+                t = item_tok[w.begin + lane];
                 toks[islot * kTok + lane] = t;
             }
             if (lane == 0) {
@@ -341,9 +341,9 @@ cudaError_t launch_score(const LaunchCtx& c, const ScoreArgs& a) {
     if (a.dtype == LOOKME_BF16)
         return launch_pdl(k3_score<__nv_bfloat16>, dim3(c.num_sms), dim3(k3::kThreads), (size_t)g.smem, c.stream,
                           (const __nv_bfloat16*)a.q, (const __nv_bfloat16*)a.keys, a.P, a.dk, a.top_k, a.scale, a.work,
-                          a.counters, a.perm, a.use_slots, a.prim_out, a.weight_out, a.status, g);
+                          a.counters, a.item_tok, a.use_slots, a.prim_out, a.weight_out, a.status, g);
     return launch_pdl(k3_score<float>, dim3(c.num_sms), dim3(k3::kThreads), (size_t)g.smem, c.stream,
-                      (const float*)a.q, (const float*)a.keys, a.P, a.dk, a.top_k, a.scale, a.work, a.counters, a.perm,
+                      (const float*)a.q, (const float*)a.keys, a.P, a.dk, a.top_k, a.scale, a.work, a.counters, a.item_tok,
                       a.use_slots, a.prim_out, a.weight_out, a.status, g);
 }
 

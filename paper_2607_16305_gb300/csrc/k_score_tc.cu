@@ -31,10 +31,10 @@
 //                item's top-k overlaps the next item's read-out): TMEM ->
 //                logits in shared memory (scaled), then top-k + softmax, one
 //                token per warp
-//   warp 18      token tiles: reads the item's token ids and query rows with
-//                plain 16-byte loads and writes them straight into the
-//                swizzled tile (small copies would each cost the copy engine
-//                as much time as a 64 KiB one)
+//   warp 18      token tiles: reads the item's token ids and copies its query
+//                rows with 16-byte cp.async straight into the swizzled tile,
+//                all of them in flight at once (bulk copies of a row would
+//                each cost the copy engine as much time as a 64 KiB one)
 // Before the grid dependency wait, the MMA issuer and the top-k run once
 // without effect, so their code is cached before the key stream starts (a
 // first instruction fetch under the full stream costs microseconds).
@@ -62,7 +62,6 @@ constexpr int kGroupWarps = 8;           // epilogue warps per item group (one t
 constexpr int kEpiWarps = 2 * kGroupWarps;
 constexpr int kBuildWarp = 2 + kEpiWarps;
 constexpr int kThreads = (3 + kEpiWarps) * 32;
-constexpr int kQBatch = 4;               // query-row chunks in flight per lane
 constexpr int kMaxStages = 14;           // ring slots (barrier arrays)
 constexpr int kBSlots = 2;               // token tiles
 constexpr int kISlots = 4;               // item metadata (scene, count, token ids)
@@ -187,7 +186,7 @@ __device__ __forceinline__ void prefetch_row_l2(const uint8_t* row, int64_t byte
 __global__ void __launch_bounds__(k3tc::kThreads, 1)
     k3_score_tc(const uint8_t* __restrict__ keys_t, int64_t block_bytes, const __nv_bfloat16* q,
                 int64_t P, int dk, int top_k, float scale, const WorkItem* work,
-                const int32_t* counters, const int32_t* perm, int64_t work_cap, int use_slots,
+                const int32_t* counters, const int32_t* item_tok, int64_t work_cap, int use_slots,
                 int32_t* __restrict__ prim_out, float* __restrict__ weight_out, uint32_t* __restrict__ status,
                 const uint8_t* keep_mask, const uint8_t* __restrict__ values, int64_t vrow_bytes,
                 const __grid_constant__ k3tc::Geometry g) {
@@ -240,11 +239,17 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
     // wait); TMEM is allocated only after it, so a CTA that holds TMEM never
     // waits on an earlier kernel.
     pdl_wait();
-    // This CTA's first work entry is read together with the count (the work
-    // array holds work_cap entries), saving a dependent round trip.
+    // This CTA's first work entry, and the token-tile warp's first token ids,
+    // are read together with the count (the work array holds work_cap
+    // entries, the token array kTok per entry), saving dependent round trips;
+    // the token ids are used only for lanes below the entry's count.
     WorkItem w0;
     w0.scene = w0.begin = w0.count = w0.slot = 0;
-    if ((int64_t)blockIdx.x < work_cap) w0 = work[blockIdx.x];
+    int32_t tok0 = 0;
+    if ((int64_t)blockIdx.x < work_cap) {
+        w0 = work[blockIdx.x];
+        if (warp == kBuildWarp && lane < kTok) tok0 = item_tok[(int64_t)blockIdx.x * kTok + lane];
+    }
     const int n_work = counters[0];
     const int G = gridDim.x;
     const int my_items = n_work > (int)blockIdx.x ? (n_work - (int)blockIdx.x + G - 1) / G : 0;
@@ -454,9 +459,10 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         for (int idx = lane; idx < kBSlots * g.b_bytes / 16; idx += 32)
             reinterpret_cast<uint4*>(btile)[idx] = make_uint4(0u, 0u, 0u, 0u);
         const int cpr = g.row_bytes / 16;  // 16-byte chunks per query row
-        const uint4* qv = reinterpret_cast<const uint4*>(q);
+        const uint8_t* qb = reinterpret_cast<const uint8_t*>(q);
+        const uint32_t bt0 = ptx::smem_u32(btile);
         WorkItem w = w0;
-        int32_t tok = lane < w.count ? perm[w.begin + lane] : 0;
+        int32_t tok = lane < w.count ? tok0 : 0;
         bool kp = keep_mask && lane < w.count && keep_mask[tok];
         bool ok = true;
         for (int i = 0; i < my_items; ++i) {
@@ -470,52 +476,43 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             if (!__shfl_sync(0xFFFFFFFFu, (int)ok, 0)) break;
             const int nb = min(w.count, kTok);
             const int total = nb * cpr;
-            uint8_t* bt = btile + bs * g.b_bytes;
-            WorkItem wn = w;
-            int32_t tokn = 0;
-            bool kpn = false;
-            for (int base = 0; base < total; base += 32 * kQBatch) {
-                uint4 v[kQBatch];
-                int jj[kQBatch], cc[kQBatch];
-#pragma unroll
-                for (int u = 0; u < kQBatch; ++u) {
-                    const int idx = base + u * 32 + lane;
-                    const bool valid = idx < total;
-                    jj[u] = valid ? idx / cpr : 0;
-                    cc[u] = valid ? idx - jj[u] * cpr : -1;
-                    const int32_t tj = __shfl_sync(0xFFFFFFFFu, tok, jj[u]);
-                    if (valid) v[u] = __ldg(qv + (int64_t)tj * cpr + cc[u]);
-                }
-                // The next work entry is read while the query rows are in flight.
-                if (base == 0 && i + 1 < my_items) wn = work[item_index(i + 1)];
-#pragma unroll
-                for (int u = 0; u < kQBatch; ++u) {
-                    if (cc[u] >= 0) {
-                        // Row j of k-block kb: 16-byte chunk c at position c ^ j (j < 8).
-                        const int j = jj[u], kb = cc[u] >> 3, c = cc[u] & 7;
-                        *reinterpret_cast<uint4*>(bt + kb * kAtomBytes + j * 128 + ((c ^ j) * 16)) = v[u];
-                    }
+            const uint32_t bt = bt0 + (uint32_t)(bs * g.b_bytes);
+            // Every query chunk of the item in flight at once, straight into the
+            // swizzled tile: row j of k-block kb, 16-byte chunk c at position c ^ j.
+            for (int base = 0; base < total; base += 32) {
+                const int idx = base + lane;
+                const int j = idx / cpr, cc = idx - j * cpr;
+                const int32_t tj = __shfl_sync(0xFFFFFFFFu, tok, j & (kTok - 1));
+                if (idx < total) {
+                    const int kb = cc >> 3, c = cc & 7;
+                    ptx::cp_async16(bt + (uint32_t)(kb * kAtomBytes + j * 128 + ((c ^ j) * 16)),
+                                    qb + (int64_t)tj * g.row_bytes + cc * 16);
                 }
             }
-            if (total == 0 && i + 1 < my_items) wn = work[item_index(i + 1)];
-            if (i + 1 < my_items) tokn = lane < wn.count ? perm[wn.begin + lane] : 0;
+            // The next item's entry and token ids are read while the rows are in flight.
+            WorkItem wn = w;
+            int32_t tokn = 0;
+            if (i + 1 < my_items) {
+                wn = work[item_index(i + 1)];
+                if (lane < kTok) tokn = item_tok[(int64_t)item_index(i + 1) * kTok + lane];
+            }
+            ptx::cp_async_wait_all();
             if (i == 0 && !__all_sync(0xFFFFFFFFu, ptx::mbar_wait(setup, 0, abort, kTimeoutNs))) break;
             ptx::fence_proxy_async_smem();  // the tile is read by the tensor core (async proxy)
             if (lane < nb) toks[ms * kTok + lane] = tok;
-            const uint32_t kb = __ballot_sync(0xFFFFFFFFu, kp);
+            const uint32_t kbits = __ballot_sync(0xFFFFFFFFu, kp);
             if (lane == 0) {
                 items[ms] = w;
-                keepbits[ms] = kb;
+                keepbits[ms] = kbits;
             }
-            if (i + 1 < my_items) kpn = keep_mask && lane < wn.count && keep_mask[tokn];
             __syncwarp();
             if (lane == 0) {
                 ptx::mbar_arrive(&ifull[ms]);
                 ptx::mbar_arrive(&bfull[bs]);
             }
             w = wn;
-            tok = tokn;
-            kp = kpn;
+            tok = lane < w.count ? tokn : 0;
+            kp = keep_mask && i + 1 < my_items && lane < w.count && keep_mask[tok];
         }
     }
 
@@ -544,7 +541,7 @@ cudaError_t launch_score_tc(const LaunchCtx& c, const void* keys_tiled, const Sc
     if (!score_tc_shape_supported(a.P, a.dk)) return cudaErrorInvalidConfiguration;
     return launch_pdl(k3_score_tc, dim3(c.num_sms), dim3(k3tc::kThreads), (size_t)g.smem, c.stream,
                       (const uint8_t*)keys_tiled, (int64_t)g.spi * k3tc::kSubBytes, (const __nv_bfloat16*)a.q, a.P,
-                      a.dk, a.top_k, a.scale, a.work, (const int32_t*)a.counters, a.perm, a.work_cap, a.use_slots, a.prim_out,
+                      a.dk, a.top_k, a.scale, a.work, (const int32_t*)a.counters, a.item_tok, a.work_cap, a.use_slots, a.prim_out,
                       a.weight_out, a.status, a.keep_mask, (const uint8_t*)a.values, a.vrow_bytes, g);
 }
 

@@ -124,7 +124,7 @@ struct lookme_table {
     void* scratch = nullptr;
     unsigned long long* best = nullptr;
     float* qnorm = nullptr;
-    int32_t* perm = nullptr;
+    int32_t* item_tok = nullptr;
     WorkItem* work = nullptr;
     int32_t* routed = nullptr;
     int32_t* counters = nullptr;  // n_work, n_routed, max bucket
@@ -213,8 +213,8 @@ lookme_status ensure_scratch(lookme_table* t, int64_t n, cudaStream_t s) {
     };
     const size_t o_best = take(cap * sizeof(unsigned long long));
     const size_t o_qnorm = take(cap * sizeof(float));
-    const size_t o_perm = take(cap * sizeof(int32_t));
     const size_t o_work = take((cap + S) * sizeof(WorkItem));
+    const size_t o_itok = take((cap + S) * kTokensPerItem * sizeof(int32_t));
     const size_t o_routed = take(S * sizeof(int32_t));
     const size_t o_counters = take(4 * sizeof(int32_t));
     const size_t o_sel = take(cap * sizeof(int32_t));
@@ -230,8 +230,8 @@ lookme_status ensure_scratch(lookme_table* t, int64_t n, cudaStream_t s) {
     t->cap = cap;
     t->best = reinterpret_cast<unsigned long long*>(b + o_best);
     t->qnorm = reinterpret_cast<float*>(b + o_qnorm);
-    t->perm = reinterpret_cast<int32_t*>(b + o_perm);
     t->work = reinterpret_cast<WorkItem*>(b + o_work);
+    t->item_tok = reinterpret_cast<int32_t*>(b + o_itok);
     t->routed = reinterpret_cast<int32_t*>(b + o_routed);
     t->counters = reinterpret_cast<int32_t*>(b + o_counters);
     t->sel = reinterpret_cast<int32_t*>(b + o_sel);
@@ -537,7 +537,7 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
     }
     if (st != LOOKME_OK) return st;
     st = launch(t, s, KID_BUCKET, [&] {
-        return launch_bucket(ctx, t->best, N, d.n_scenes, scene_out, t->perm, t->work, t->routed, t->counters,
+        return launch_bucket(ctx, t->best, N, d.n_scenes, scene_out, t->item_tok, t->work, t->routed, t->counters,
                              gate);
     });
     if (st != LOOKME_OK) return st;
@@ -559,7 +559,7 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
     a.work = t->work;
     a.work_cap = t->cap + d.n_scenes;
     a.counters = t->counters;
-    a.perm = t->perm;
+    a.item_tok = t->item_tok;
     a.use_slots = staged ? 1 : 0;
     a.prim_out = prim_out;
     a.weight_out = weight_out;
