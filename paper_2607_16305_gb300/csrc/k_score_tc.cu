@@ -158,22 +158,44 @@ __device__ __noinline__ void mma_kblock(uint32_t live, uint32_t d, uint64_t ad, 
 
 // Top-k + softmax of one token over logits at stride kZStride; a single copy
 // serves the warm-up call (prim_out == nullptr: nothing is written) and the
-// real ones.  The common shape (N_p <= 256, top_k <= 8) has a function of its
-// own, so that the larger variants' registers do not weigh on it.
+// real ones.  Each variant is a function of its own, so that no variant's
+// registers weigh on another (one function holding them all spills).
 // Each returns the lane's selected primitive (lanes < top_k, first 32), else -1.
-__device__ __noinline__ int topk_small(const float* z, int64_t P, int top_k, int lane, int64_t t,
-                                       int32_t* prim_out, float* weight_out) {
-    if (P <= 64) return k3::topk_token_pop<2, 8>(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
-    return k3::topk_token_pop<8, 8>(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
+template <int PPL, int L>
+__device__ __noinline__ int topk_pop_fn(const float* z, int64_t P, int top_k, int lane, int64_t t, int32_t* prim_out,
+                                        float* weight_out) {
+    return k3::topk_token_pop<PPL, L>(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
 }
-__device__ __noinline__ int topk_large(const float* z, int64_t P, int top_k, int lane, int64_t t,
-                                       int32_t* prim_out, float* weight_out) {
-    return k3::topk_any(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
+template <int PPL>
+__device__ __noinline__ int topk_regs_fn(const float* z, int64_t P, int top_k, int lane, int64_t t,
+                                         int32_t* prim_out, float* weight_out) {
+    return k3::topk_token_regs<PPL>(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
 }
+__device__ __noinline__ int topk_scan_fn(const float* z, int64_t P, int top_k, int lane, int64_t t, int32_t* prim_out,
+                                         float* weight_out) {
+    return k3::topk_token(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
+}
+// The variant choice of k3::topk_any.
 __device__ __forceinline__ int topk_item(const float* z, int64_t P, int top_k, int lane, int64_t t,
                                          int32_t* prim_out, float* weight_out) {
-    if (P <= 256 && top_k <= 8) return topk_small(z, P, top_k, lane, t, prim_out, weight_out);
-    return topk_large(z, P, top_k, lane, t, prim_out, weight_out);
+    if (top_k <= 8) {
+        if (P <= 64) return topk_pop_fn<2, 8>(z, P, top_k, lane, t, prim_out, weight_out);
+        if (P <= 256) return topk_pop_fn<8, 8>(z, P, top_k, lane, t, prim_out, weight_out);
+        if (P <= 512) return topk_pop_fn<16, 8>(z, P, top_k, lane, t, prim_out, weight_out);
+        if (P <= 1024) return topk_pop_fn<32, 8>(z, P, top_k, lane, t, prim_out, weight_out);
+        return topk_scan_fn(z, P, top_k, lane, t, prim_out, weight_out);
+    }
+    if (top_k <= 16 && P <= 1024) {
+        if (P <= 512) return topk_pop_fn<16, 16>(z, P, top_k, lane, t, prim_out, weight_out);
+        return topk_pop_fn<32, 16>(z, P, top_k, lane, t, prim_out, weight_out);
+    }
+    if (P <= 32) return topk_regs_fn<1>(z, P, top_k, lane, t, prim_out, weight_out);
+    if (P <= 64) return topk_regs_fn<2>(z, P, top_k, lane, t, prim_out, weight_out);
+    if (P <= 128) return topk_regs_fn<4>(z, P, top_k, lane, t, prim_out, weight_out);
+    if (P <= 256) return topk_regs_fn<8>(z, P, top_k, lane, t, prim_out, weight_out);
+    if (P <= 512) return topk_regs_fn<16>(z, P, top_k, lane, t, prim_out, weight_out);
+    if (P <= 1024) return topk_regs_fn<32>(z, P, top_k, lane, t, prim_out, weight_out);
+    return topk_scan_fn(z, P, top_k, lane, t, prim_out, weight_out);
 }
 
 // Pull one value row into L2 (128-byte lines, no register result).

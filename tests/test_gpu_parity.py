@@ -104,7 +104,7 @@ def run_case(o, lookme_lib, w, *, sample=None, give_centroids=True, bias_scale=0
     res["mask_ties"] = mask_ties
     res.pop("wref")
     if report is not None:
-        report.update(res, stats=stats)
+        report.update(res, stats=stats, scene=gscene)
     print(f"{w.name}: {res} stats={stats}")
     return res
 
@@ -262,6 +262,34 @@ def test_cuda_core_variants(oracle, lookme_lib, monkeypatch, case):
     else:
         w = W.small("s6_simt", **dict(SMALL_CASES)["s6"])
     run_case(oracle, lookme_lib, w)
+
+
+@pytest.mark.parametrize("name", ["s1", "s2", "s4", "s5", "s6", "s7", "layers"])
+def test_lookup_inject_small_against_oracle(oracle, lookme_lib, name):
+    """lookme_lookup_inject on bf16 tables (gate decided beside the
+    bucketing, level 2 on the tensor cores, injection of the kept tokens)
+    against the oracle, over the small shapes and three layers."""
+    kw = dict(SMALL_CASES).get(name) or dict(n_tokens=256, n_scenes=16, n_prims=32, d_key=64, d_value=128, top_k=4,
+                                           keep_ratio=0.5)
+    w = W.small(f"lif_{name}", dtype="bf16", **kw)
+    run_case(oracle, lookme_lib, w, fused=True, n_layers=3 if name == "layers" else None)
+
+
+@pytest.mark.parametrize("extra", [0, 1])
+def test_lookup_inject_many_items(oracle, lookme_lib, extra):
+    """32 tokens per SM (and one more) spread over 32,768 scenes, so most
+    tokens are alone in their scene and every level-2 CTA takes about 30 work
+    items, with the work-list counters against the routed scenes."""
+    n_sms = torch.cuda.get_device_properties(0).multi_processor_count
+    n = n_sms * 32 + extra
+    w = W.small(f"limit_{extra}", dtype="bf16", n_tokens=n, n_scenes=32768, n_prims=16, d_key=32, d_value=16,
+                top_k=4, keep_ratio=0.25)
+    rep = {}
+    run_case(oracle, lookme_lib, w, fused=True, report=rep)
+    st = rep["stats"]
+    counts = np.bincount(rep["scene"], minlength=w.n_scenes)
+    assert st["n_routed_scenes"] == int((counts > 0).sum())
+    assert st["n_work_items"] == int(((counts + 7) // 8).sum())
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "fp32"])
