@@ -22,9 +22,12 @@
 // an SM spends about the same time on a 16 KiB and a 64 KiB copy, so large
 // copies are what lets one CTA per SM pull its share of HBM bandwidth.
 //
-// One CTA per SM, static share of the work list (items b, b + G, ...):
-//   warp 0       producer: reads each item's work entry and streams the
-//                scene's key block through the ring (bulk copies only)
+// One CTA per SM.  CTA b's first item is work entry b; the entries from G on
+// are taken one at a time from a shared counter as CTAs progress (one item
+// ahead), so the CTAs that run ahead take the last items:
+//   warp 0       producer: takes the item indices, passes them to warp 18,
+//                reads each item's work entry and streams the scene's key
+//                block through the ring (bulk copies only)
 //   warp 1       one thread issues tcgen05.mma, N-tile by N-tile, into the
 //                two TMEM buffers
 //   warps 2..17  epilogue, two groups of eight taking alternate items (so one
@@ -65,6 +68,7 @@ constexpr int kThreads = (3 + kEpiWarps) * 32;
 constexpr int kMaxStages = 14;           // ring slots (barrier arrays)
 constexpr int kBSlots = 2;               // token tiles
 constexpr int kISlots = 4;               // item metadata (scene, count, token ids)
+constexpr int kSeq = 4;                  // item indices passed from the producer to the token-tile warp
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 constexpr int kSmemLimit = 227 * 1024;
 
@@ -113,8 +117,8 @@ inline Geometry geometry(int64_t P, int dk) {
     g.off_b = g.n_stages * g.slot_bytes;
     g.off_z = g.off_b + kBSlots * g.b_bytes;
     g.off_bar = g.off_z + 2 * g.zbytes;
-    g.off_meta = g.off_bar + (2 * kMaxStages + 2 * kBSlots + 2 * kISlots + 4 + 2 + 1 + 2) * 8;
-    g.smem = g.off_meta + kISlots * ((int)sizeof(WorkItem) + kTok * 4 + 4) + 16 + 1024;
+    g.off_meta = g.off_bar + (2 * kMaxStages + 2 * kBSlots + 2 * kISlots + 4 + 2 + 1 + 2 + 2 * kSeq) * 8;
+    g.smem = g.off_meta + kISlots * ((int)sizeof(WorkItem) + kTok * 4 + 4) + 16 + kSeq * 4 + 1024;
     return g;
 }
 
@@ -208,7 +212,7 @@ __device__ __forceinline__ void prefetch_row_l2(const uint8_t* row, int64_t byte
 __global__ void __launch_bounds__(k3tc::kThreads, 1)
     k3_score_tc(const uint8_t* __restrict__ keys_t, int64_t block_bytes, const __nv_bfloat16* q,
                 int64_t P, int dk, int top_k, float scale, const WorkItem* work,
-                const int32_t* counters, const int32_t* item_tok, int64_t work_cap, int use_slots,
+                int32_t* counters, const int32_t* item_tok, int64_t work_cap, int use_slots,
                 int32_t* __restrict__ prim_out, float* __restrict__ weight_out, uint32_t* __restrict__ status,
                 const uint8_t* keep_mask, const uint8_t* __restrict__ values, int64_t vrow_bytes,
                 const __grid_constant__ k3tc::Geometry g) {
@@ -233,11 +237,16 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
     uint64_t* drain = tempty + 2;
     uint64_t* setup = drain + 1;      // the other barriers are initialised (thread 0)
     uint64_t* tmem_ready = setup + 1; // the TMEM address is in tmem_slot (warp 1)
+    // Item j >= 1 of the CTA (item 0 is entry b) is queue entry j - 1: its index
+    // is in seq[(j - 1) % kSeq], phase (j - 1) / kSeq of seqfull / seqempty.
+    uint64_t* seqfull = tmem_ready + 1;
+    uint64_t* seqempty = seqfull + kSeq;
     WorkItem* items = reinterpret_cast<WorkItem*>(smem + g.off_meta);
     int32_t* toks = reinterpret_cast<int32_t*>(items + kISlots);
     uint32_t* keepbits = reinterpret_cast<uint32_t*>(toks + kISlots * kTok);  // gate of the item's tokens
     uint32_t* tmem_slot = keepbits + kISlots;
     volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    int32_t* seq = reinterpret_cast<int32_t*>(tmem_slot + 4);  // item indices; -1 ends the list
 
     const int tid = threadIdx.x, lane = tid % 32, warp = tid / 32;
     pdl_trigger();
@@ -274,8 +283,10 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
     }
     const int n_work = counters[0];
     const int G = gridDim.x;
-    const int my_items = n_work > (int)blockIdx.x ? (n_work - (int)blockIdx.x + G - 1) / G : 0;
-    if (my_items == 0) return;  // uniform for the CTA: nothing allocated yet
+    // Item 0 of CTA b is work entry b; the entries from G on are taken one at
+    // a time from a shared counter (reset by the bucketing kernel) as the CTA
+    // progresses, so CTAs that run ahead take more of the last items.
+    if (n_work <= (int)blockIdx.x) return;  // uniform for the CTA: nothing allocated yet
     if (tid == 0) {
         for (int i = 0; i < g.n_stages; ++i) {
             ptx::mbar_init(&full[i], 1);
@@ -291,11 +302,14 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         }
         for (int i = 0; i < 4; ++i) ptx::mbar_init(&dready[i], 1);
         for (int i = 0; i < 2; ++i) ptx::mbar_init(&tempty[i], kGroupWarps);
+        for (int i = 0; i < kSeq; ++i) {
+            ptx::mbar_init(&seqfull[i], 1);
+            ptx::mbar_init(&seqempty[i], 1);
+        }
         ptx::mbar_init(drain, 1);
         ptx::fence_mbar_init();
         ptx::mbar_arrive(setup);
     }
-    auto item_index = [&](int i) { return (int)blockIdx.x + i * G; };
     // N-tile nt: its first sub-block, its sub-block count (1 or 2) and its N.
     auto nt_base = [&](int nt) { return nt * 2 * g.nkb; };
     auto nt_subs = [&](int nt) { return (nt == g.nnt - 1 && (g.ntile & 1)) ? 1 : 2; };
@@ -350,13 +364,31 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
                 }
             }
         };
-        // The work entry of the next item is loaded while this one's copies go out.
-        WorkItem w = w0;
-        for (int i = 0; i < my_items && ok; ++i) {
-            WorkItem wn = w;
-            if (i + 1 < my_items) wn = work[item_index(i + 1)];
-            issue_stages(w, 0, g.chunks);
-            w = wn;
+        // Item i + 1's index is taken as item i's first copy goes out and passed
+        // to the token-tile warp through seq (-1: no more items) before the
+        // item's other copies, which may wait for ring slots that only item i's
+        // token tile frees; its work entry is read before item i + 1's first copy.
+        WorkItem w = w0, w_next = w0;
+        for (int i = 0; ok; ++i) {
+            int taken = 0;
+            if (lane == 0) taken = G + atomicAdd(counters + 3, 1);
+            issue_stages(w, 0, 1);
+            int nxt = -1;
+            if (lane == 0 && ok) {
+                nxt = taken < n_work ? taken : -1;
+                const int qs = i % kSeq;  // item i + 1: queue entry i
+                ok = ptx::mbar_wait(&seqempty[qs], ((i / kSeq) & 1) ^ 1, abort, kTimeoutNs);
+                if (ok) {
+                    seq[qs] = nxt;
+                    ptx::mbar_arrive(&seqfull[qs]);
+                }
+            }
+            ok = __shfl_sync(0xFFFFFFFFu, (int)ok, 0) != 0;
+            nxt = __shfl_sync(0xFFFFFFFFu, nxt, 0);
+            if (ok && nxt >= 0) w_next = work[nxt];
+            issue_stages(w, 1, g.chunks);
+            if (!ok || nxt < 0) break;
+            w = w_next;
         }
         if (!ok && lane == 0) {
             // Let every copy still in flight land before the CTA can exit.
@@ -371,9 +403,10 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             uint32_t phase = 0;
             int qn = 0;  // N-tiles issued (D buffer qn & 1)
             bool ok = true;
-            for (int i = 0; i < my_items && ok; ++i) {
+            for (int i = 0; ok; ++i) {
                 const int bs = i % kBSlots;
                 if (!(ok = ptx::mbar_wait(&bfull[bs], (i / kBSlots) & 1, abort, kTimeoutNs))) break;
+                if (items[i % kISlots].count < 0) break;  // the end of the CTA's list
                 ptx::tc_fence_after();
                 const uint64_t ad0 = sw128_desc(a_tiles + (uint32_t)(bs * g.b_bytes), 0);
                 int cur_chunk = -1;
@@ -426,11 +459,12 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         const int eg = e % kGroupWarps;   // token of the top-k, column slice of the read-out
         const int quarter = warp & 3;     // TMEM lanes this warp may access
         float* zg = zs + grp * (g.zbytes / 4);
-        for (int i = grp; i < my_items; i += 2) {
+        for (int i = grp;; i += 2) {
             const int ms = i % kISlots;
             bool ok = __all_sync(0xFFFFFFFFu, ptx::mbar_wait(&ifull[ms], (i / kISlots) & 1, abort, kTimeoutNs));
             // Also orders this item's logit writes after the group's top-k of its previous item.
             if (k3tc::group_sync_or(grp, !ok || *abort)) break;
+            if (items[ms].count < 0) break;  // the end of the CTA's list (uniform)
             const int nb = min(items[ms].count, kTok);
             for (int nt = 0; nt < g.nnt; ++nt) {
                 const int qn = i * g.nnt + nt, buf = qn & 1;
@@ -487,7 +521,10 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         int32_t tok = lane < w.count ? tok0 : 0;
         bool kp = keep_mask && lane < w.count && keep_mask[tok];
         bool ok = true;
-        for (int i = 0; i < my_items; ++i) {
+        // The items until the producer's -1, then two end markers (count -1):
+        // one for each epilogue group, the first also read by the MMA issuer.
+        int ends = 0;
+        for (int i = 0; ends < 2; ++i) {
             const int ms = i % kISlots, bs = i % kBSlots;
             // The first item's slots are free by construction: its query rows are
             // loaded before this warp touches any barrier (and before the key
@@ -496,6 +533,15 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
                 ok = ptx::mbar_wait(&iempty[ms], ((i / kISlots) & 1) ^ 1, abort, kTimeoutNs) &&
                      ptx::mbar_wait(&bempty[bs], ((i / kBSlots) & 1) ^ 1, abort, kTimeoutNs);
             if (!__shfl_sync(0xFFFFFFFFu, (int)ok, 0)) break;
+            if (w.count < 0) {
+                if (lane == 0) {
+                    items[ms] = w;
+                    ptx::mbar_arrive(&ifull[ms]);
+                    if (ends == 0) ptx::mbar_arrive(&bfull[bs]);
+                }
+                ++ends;
+                continue;
+            }
             const int nb = min(w.count, kTok);
             const int total = nb * cpr;
             const uint32_t bt = bt0 + (uint32_t)(bs * g.b_bytes);
@@ -511,13 +557,40 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
                                     qb + (int64_t)tj * g.row_bytes + cc * 16);
                 }
             }
-            // The next item's entry and token ids are read while the rows are in flight.
-            WorkItem wn = w;
+            // The next item's index (queue entry i, which the producer publishes as
+            // item i's first copy goes out), its work entry and token ids: read
+            // while the rows are in flight when the index is already there, else
+            // once this item is published (this item never waits for the next).
+            const int qs = i % kSeq;
+            WorkItem wn;
+            wn.scene = wn.begin = wn.slot = 0;
+            wn.count = -1;
             int32_t tokn = 0;
-            if (i + 1 < my_items) {
-                wn = work[item_index(i + 1)];
-                if (lane < kTok) tokn = item_tok[(int64_t)item_index(i + 1) * kTok + lane];
-            }
+            bool have = false;
+            auto take_next = [&](bool block) {
+                int nidx = -1, got = 0;
+                if (lane == 0) {
+                    got = block ? ptx::mbar_wait(&seqfull[qs], (i / kSeq) & 1, abort, kTimeoutNs)
+                                : ptx::mbar_try_wait(&seqfull[qs], (i / kSeq) & 1);
+                    if (got) {
+                        nidx = seq[qs];
+                        ptx::mbar_arrive(&seqempty[qs]);
+                        if (nidx >= n_work) {  // not an index the producer can take: stop the CTA
+                            *abort = 1;
+                            got = 0;
+                            nidx = -1;
+                        }
+                    }
+                }
+                got = __shfl_sync(0xFFFFFFFFu, got, 0);
+                nidx = __shfl_sync(0xFFFFFFFFu, nidx, 0);
+                if (got && nidx >= 0) {
+                    wn = work[nidx];
+                    if (lane < kTok) tokn = item_tok[(int64_t)nidx * kTok + lane];
+                }
+                return got != 0;
+            };
+            have = take_next(false);
             ptx::cp_async_wait_all();
             if (i == 0 && !__all_sync(0xFFFFFFFFu, ptx::mbar_wait(setup, 0, abort, kTimeoutNs))) break;
             ptx::fence_proxy_async_smem();  // the tile is read by the tensor core (async proxy)
@@ -532,9 +605,10 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
                 ptx::mbar_arrive(&ifull[ms]);
                 ptx::mbar_arrive(&bfull[bs]);
             }
+            if (!have && !take_next(true)) break;
             w = wn;
             tok = lane < w.count ? tokn : 0;
-            kp = keep_mask && i + 1 < my_items && lane < w.count && keep_mask[tok];
+            kp = keep_mask && lane < w.count && keep_mask[tok];
         }
     }
 
@@ -563,7 +637,7 @@ cudaError_t launch_score_tc(const LaunchCtx& c, const void* keys_tiled, const Sc
     if (!score_tc_shape_supported(a.P, a.dk)) return cudaErrorInvalidConfiguration;
     return launch_pdl(k3_score_tc, dim3(c.num_sms), dim3(k3tc::kThreads), (size_t)g.smem, c.stream,
                       (const uint8_t*)keys_tiled, (int64_t)g.spi * k3tc::kSubBytes, (const __nv_bfloat16*)a.q, a.P,
-                      a.dk, a.top_k, a.scale, a.work, (const int32_t*)a.counters, a.item_tok, a.work_cap, a.use_slots, a.prim_out,
+                      a.dk, a.top_k, a.scale, a.work, a.counters, a.item_tok, a.work_cap, a.use_slots, a.prim_out,
                       a.weight_out, a.status, a.keep_mask, (const uint8_t*)a.values, a.vrow_bytes, g);
 }
 
