@@ -169,10 +169,18 @@ struct ScoreArgs {
     float* weight_out;
     uint32_t* status;
     // Optional (tcgen05 level 2): the injection gate decided beside the
-    // bucketing; the value rows of kept tokens are prefetched into L2.
-    const uint8_t* keep_mask;
+    // bucketing, as each kept token's slot in the kept-id list (-1: not
+    // kept); the value rows (and the first layer's hidden row) of kept tokens
+    // are prefetched into L2.
+    const int32_t* selpos;
     const void* values;   // [S][P][d_v], device memory
     int64_t vrow_bytes;   // d_v * element size
+    const void* hidden0;  // the first layer's hidden states (prefetch only), or null
+    // Optional: the injection records of kept tokens at their slots: token id,
+    // and top_k value rows (scene * N_p + p) and weights (stride top_k).
+    int32_t* rec_t;
+    int32_t* rec_row;
+    float* rec_w;
 };
 cudaError_t launch_score(const LaunchCtx& c, const ScoreArgs& a);
 // Whether the level-2 kernel's shared-memory plan fits this table shape.
@@ -190,6 +198,7 @@ struct GateSpec {
     const float* priority;
     uint8_t* mask;
     int32_t* sel;
+    int32_t* selpos;  // optional: per token its slot sel_base + rank when kept, else -1
     int64_t off[kMaxGateSegments + 1];
     int64_t sel_base[kMaxGateSegments];
 };
@@ -227,6 +236,11 @@ struct InjectArgs {
     void* hidden[LOOKME_MAX_LAYERS];
 };
 cudaError_t launch_inject(const LaunchCtx& c, const InjectArgs& a);
+// K4 from the records the tcgen05 level-2 kernel wrote (ScoreArgs::rec_*):
+// one CTA per kept slot, every load it needs issued in one round trip.
+constexpr int kRecMaxTopK = 16;
+cudaError_t launch_inject_records(const LaunchCtx& c, const InjectArgs& a, const int32_t* rec_t,
+                                  const int32_t* rec_row, const float* rec_w);
 // K5 + K4 in one kernel (one CTA per token) for segments of at most
 // kFusedMaxSegment tokens when the kept-id list is not requested.
 constexpr int64_t kFusedMaxSegment = 8192;

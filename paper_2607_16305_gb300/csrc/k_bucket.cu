@@ -18,7 +18,8 @@
 // With a gate, CTAs 1.. compute the injection gate meanwhile, eight tokens
 // per CTA (one per warp; a light load per SM so they finish within the
 // bucketing): rank_t = #{ j in segment : pi_j > pi_t, or pi_j == pi_t and
-// j < t }, kept iff rank_t < r, the kept ones listed at sel[sel_base + rank_t].
+// j < t }, kept iff rank_t < r, the kept ones listed at sel[sel_base + rank_t]
+// (and, optionally, that slot recorded per token in selpos, -1 if not kept).
 // Each CTA stages the priorities its tokens' segments span in shared memory
 // once.  This runs before the level-2 key stream, whose copies would
 // otherwise queue every small load behind them.
@@ -91,6 +92,7 @@ __device__ void gate_block(const GateSpec& gs, float* buf, int cap) {
     if (lane == 0) {
         gs.mask[t] = (uint8_t)keep;
         if (keep) gs.sel[gs.sel_base[sg] + rank] = (int32_t)t;
+        if (gs.selpos) gs.selpos[t] = keep ? (int32_t)(gs.sel_base[sg] + rank) : -1;
     }
 }
 // Exclusive block-wide scan of two counters at once.
@@ -147,7 +149,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = tid; s < S; s += kThreads) cnt[s] = 0;
     if (tid == 0) max_bucket = 0;
     __syncthreads();
-    for (int64_t t = tid; t < N; t += kThreads) {
+    // The scenes of a thread's first kCache tokens stay in registers for the
+    // second sweep (no second read of the keys).
+    constexpr int kCache = 4;
+    int32_t sc[kCache];
+    {
+        unsigned long long key[kCache];
+#pragma unroll
+        for (int u = 0; u < kCache; ++u) {
+            const int64_t t = tid + (int64_t)u * kThreads;
+            key[u] = t < N ? best[t] : 0ull;
+        }
+#pragma unroll
+        for (int u = 0; u < kCache; ++u) {
+            const int64_t t = tid + (int64_t)u * kThreads;
+            sc[u] = unpack_scene(key[u], S);
+            if (t < N) {
+                scene_out[t] = sc[u];
+                atomicAdd(&cnt[sc[u]], 1);
+            }
+        }
+    }
+    for (int64_t t = tid + (int64_t)kCache * kThreads; t < N; t += kThreads) {
         const int32_t s = unpack_scene(best[t], S);
         scene_out[t] = s;
         atomicAdd(&cnt[s], 1);
@@ -193,10 +216,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         counters[2] = max_bucket;
         counters[3] = 0;  // level-2 work-taking counter
     }
-    for (int64_t t = tid; t < N; t += kThreads) {
+    // A scene's k-th token lands in its item k / 8, lane k % 8; the keys are
+    // cleared for the next call's argmax.
+#pragma unroll
+    for (int u = 0; u < kCache; ++u) {
+        const int64_t t = tid + (int64_t)u * kThreads;
+        if (t < N) {
+            best[t] = 0ull;
+            const int pos = atomicAdd(&cnt[sc[u]], 1);
+            item_tok[pos] = (int32_t)t;
+        }
+    }
+    for (int64_t t = tid + (int64_t)kCache * kThreads; t < N; t += kThreads) {
         const int32_t s = unpack_scene(best[t], S);
-        best[t] = 0ull;  // ready for the next call's argmax
-        // A scene's k-th token lands in its item k / 8, lane k % 8.
+        best[t] = 0ull;
         const int pos = atomicAdd(&cnt[s], 1);
         item_tok[pos] = (int32_t)t;
     }

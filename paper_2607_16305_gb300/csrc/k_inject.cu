@@ -290,6 +290,56 @@ cudaError_t launch_select_inject(const LaunchCtx& c, const InjectArgs& a, const 
     return launch_pdl(k45_select_inject<float>, dim3(grid), dim3(k45::kThreads), 0, c.stream, p, sp);
 }
 
+// K4 from level-2 records: CTA b injects the token of kept slot b, whose id,
+// value rows and weights the level-2 kernel wrote at slot b, so one round trip
+// brings everything the value-row and hidden-row loads need.
+template <typename T>
+__global__ void __launch_bounds__(k4::kThreads) k4_inject_records(const __grid_constant__ k4::Params p,
+                                                                   const int32_t* rec_t, const int32_t* rec_row,
+                                                                   const float* rec_w) {
+    __shared__ const uint4* rows[kRecMaxTopK];
+    __shared__ float w[kRecMaxTopK];
+    pdl_trigger();
+    pdl_wait();
+    const int64_t b = blockIdx.x;
+    const int64_t t = rec_t[b];  // every thread, together with the rows and weights
+    const int j = threadIdx.x;
+    if (j < p.top_k) {
+        const int64_t r = min(max((int64_t)rec_row[b * p.top_k + j], (int64_t)0), p.S * p.P - 1);
+        rows[j] = reinterpret_cast<const uint4*>(reinterpret_cast<const T*>(p.values) + r * p.dv);
+        w[j] = rec_w[b * p.top_k + j];
+    }
+    __syncthreads();
+    accumulate_store<T>(p, t, rows, w);
+}
+
+cudaError_t launch_inject_records(const LaunchCtx& c, const InjectArgs& a, const int32_t* rec_t,
+                                  const int32_t* rec_row, const float* rec_w) {
+    if (a.n_sel == 0) return cudaSuccess;
+    if (a.top_k > kRecMaxTopK) return cudaErrorInvalidValue;
+    k4::Params p;
+    p.values = a.values;
+    p.P = a.P;
+    p.dv = a.dv;
+    p.top_k = a.top_k;
+    p.scene = a.scene;
+    p.prim = a.prim;
+    p.weight = a.weight;
+    p.sel = a.sel;
+    p.N = a.N;
+    p.S = a.S;
+    p.n_layers = a.n_layers;
+    for (int l = 0; l < a.n_layers; ++l) p.hidden[l] = a.hidden[l];
+    const int chunks = a.dv / (a.dtype == LOOKME_BF16 ? 8 : 4);
+    int threads = (chunks + 31) / 32 * 32;
+    if (threads > k4::kThreads) threads = k4::kThreads;
+    if (a.dtype == LOOKME_BF16)
+        return launch_pdl(k4_inject_records<__nv_bfloat16>, dim3((unsigned)a.n_sel), dim3(threads), 0, c.stream, p,
+                          rec_t, rec_row, rec_w);
+    return launch_pdl(k4_inject_records<float>, dim3((unsigned)a.n_sel), dim3(threads), 0, c.stream, p, rec_t,
+                      rec_row, rec_w);
+}
+
 cudaError_t launch_inject(const LaunchCtx& c, const InjectArgs& a) {
     if (a.n_sel == 0) return cudaSuccess;
     k4::Params p;

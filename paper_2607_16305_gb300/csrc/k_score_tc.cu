@@ -118,7 +118,7 @@ inline Geometry geometry(int64_t P, int dk) {
     g.off_z = g.off_b + kBSlots * g.b_bytes;
     g.off_bar = g.off_z + 2 * g.zbytes;
     g.off_meta = g.off_bar + (2 * kMaxStages + 2 * kBSlots + 2 * kISlots + 4 + 2 + 1 + 2 + 2 * kSeq) * 8;
-    g.smem = g.off_meta + kISlots * ((int)sizeof(WorkItem) + kTok * 4 + 4) + 16 + kSeq * 4 + 1024;
+    g.smem = g.off_meta + kISlots * ((int)sizeof(WorkItem) + kTok * 4 + 4) + 16 + kSeq * 4 + kISlots * kTok * 4 + 1024;
     return g;
 }
 
@@ -164,23 +164,23 @@ __device__ __noinline__ void mma_kblock(uint32_t live, uint32_t d, uint64_t ad, 
 // serves the warm-up call (prim_out == nullptr: nothing is written) and the
 // real ones.  Each variant is a function of its own, so that no variant's
 // registers weigh on another (one function holding them all spills).
-// Each returns the lane's selected primitive (lanes < top_k, first 32), else -1.
+// Each returns the lane's selected primitive and its weight (lanes < top_k, first 32).
 template <int PPL, int L>
-__device__ __noinline__ int topk_pop_fn(const float* z, int64_t P, int top_k, int lane, int64_t t, int32_t* prim_out,
+__device__ __noinline__ k3::TopkLane topk_pop_fn(const float* z, int64_t P, int top_k, int lane, int64_t t, int32_t* prim_out,
                                         float* weight_out) {
     return k3::topk_token_pop<PPL, L>(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
 }
 template <int PPL>
-__device__ __noinline__ int topk_regs_fn(const float* z, int64_t P, int top_k, int lane, int64_t t,
+__device__ __noinline__ k3::TopkLane topk_regs_fn(const float* z, int64_t P, int top_k, int lane, int64_t t,
                                          int32_t* prim_out, float* weight_out) {
     return k3::topk_token_regs<PPL>(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
 }
-__device__ __noinline__ int topk_scan_fn(const float* z, int64_t P, int top_k, int lane, int64_t t, int32_t* prim_out,
+__device__ __noinline__ k3::TopkLane topk_scan_fn(const float* z, int64_t P, int top_k, int lane, int64_t t, int32_t* prim_out,
                                          float* weight_out) {
     return k3::topk_token(z, P, top_k, lane, t, prim_out, weight_out, kZStride);
 }
 // The variant choice of k3::topk_any.
-__device__ __forceinline__ int topk_item(const float* z, int64_t P, int top_k, int lane, int64_t t,
+__device__ __forceinline__ k3::TopkLane topk_item(const float* z, int64_t P, int top_k, int lane, int64_t t,
                                          int32_t* prim_out, float* weight_out) {
     if (top_k <= 8) {
         if (P <= 64) return topk_pop_fn<2, 8>(z, P, top_k, lane, t, prim_out, weight_out);
@@ -214,7 +214,9 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
                 int64_t P, int dk, int top_k, float scale, const WorkItem* work,
                 int32_t* counters, const int32_t* item_tok, int64_t work_cap, int use_slots,
                 int32_t* __restrict__ prim_out, float* __restrict__ weight_out, uint32_t* __restrict__ status,
-                const uint8_t* keep_mask, const uint8_t* __restrict__ values, int64_t vrow_bytes,
+                const int32_t* selpos, const uint8_t* __restrict__ values, int64_t vrow_bytes,
+                const uint8_t* hidden0, int32_t* __restrict__ rec_t, int32_t* __restrict__ rec_row,
+                float* __restrict__ rec_w,
                 const __grid_constant__ k3tc::Geometry g) {
     using namespace k3tc;
     extern __shared__ uint8_t smem_raw[];
@@ -247,6 +249,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
     uint32_t* tmem_slot = keepbits + kISlots;
     volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int32_t* seq = reinterpret_cast<int32_t*>(tmem_slot + 4);  // item indices; -1 ends the list
+    int32_t* tpos = seq + kSeq;  // the item's tokens' kept-list slots (-1: not kept)
 
     const int tid = threadIdx.x, lane = tid % 32, warp = tid / 32;
     pdl_trigger();
@@ -501,10 +504,23 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             }
             if (k3tc::group_sync_or(grp, *abort)) break;  // all logits of the item are in shared memory
             if (eg < nb) {
-                const int pj = k3tc::topk_item(zg + eg, P, top_k, lane, toks[ms * kTok + eg], prim_out, weight_out);
-                // A kept token's value rows are read by the injection next: start them now.
-                if (keep_mask && pj >= 0 && ((keepbits[ms] >> eg) & 1u))
-                    k3tc::prefetch_row_l2(values + ((int64_t)items[ms].scene * P + pj) * vrow_bytes, vrow_bytes);
+                const int64_t t = toks[ms * kTok + eg];
+                const k3::TopkLane r = k3tc::topk_item(zg + eg, P, top_k, lane, t, prim_out, weight_out);
+                if ((keepbits[ms] >> eg) & 1u) {
+                    // A kept token: its record for the injection kernel, and its value
+                    // rows and hidden row (read by that kernel next) into L2 now.
+                    const int64_t row = (int64_t)items[ms].scene * P + r.p;
+                    if (rec_t) {
+                        const int pos = tpos[ms * kTok + eg];
+                        if (lane < top_k) {
+                            rec_row[(int64_t)pos * top_k + lane] = (int32_t)row;
+                            rec_w[(int64_t)pos * top_k + lane] = r.w;
+                        }
+                        if (lane == 0) rec_t[pos] = (int32_t)t;
+                    }
+                    if (r.p >= 0) k3tc::prefetch_row_l2(values + row * vrow_bytes, vrow_bytes);
+                    if (hidden0 && lane == 0) k3tc::prefetch_row_l2(hidden0 + t * vrow_bytes, vrow_bytes);
+                }
             }
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&iempty[ms]);
@@ -519,7 +535,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         const uint32_t bt0 = ptx::smem_u32(btile);
         WorkItem w = w0;
         int32_t tok = lane < w.count ? tok0 : 0;
-        bool kp = keep_mask && lane < w.count && keep_mask[tok];
+        int32_t kpos = (selpos && lane < w.count) ? selpos[tok] : -1;
         bool ok = true;
         // The items until the producer's -1, then two end markers (count -1):
         // one for each epilogue group, the first also read by the MMA issuer.
@@ -595,7 +611,8 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             if (i == 0 && !__all_sync(0xFFFFFFFFu, ptx::mbar_wait(setup, 0, abort, kTimeoutNs))) break;
             ptx::fence_proxy_async_smem();  // the tile is read by the tensor core (async proxy)
             if (lane < nb) toks[ms * kTok + lane] = tok;
-            const uint32_t kbits = __ballot_sync(0xFFFFFFFFu, kp);
+            const uint32_t kbits = __ballot_sync(0xFFFFFFFFu, kpos >= 0);
+            if (lane < nb) tpos[ms * kTok + lane] = kpos;
             if (lane == 0) {
                 items[ms] = w;
                 keepbits[ms] = kbits;
@@ -608,7 +625,7 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
             if (!have && !take_next(true)) break;
             w = wn;
             tok = lane < w.count ? tokn : 0;
-            kp = keep_mask && lane < w.count && keep_mask[tok];
+            kpos = (selpos && lane < w.count) ? selpos[tok] : -1;
         }
     }
 
@@ -638,7 +655,8 @@ cudaError_t launch_score_tc(const LaunchCtx& c, const void* keys_tiled, const Sc
     return launch_pdl(k3_score_tc, dim3(c.num_sms), dim3(k3tc::kThreads), (size_t)g.smem, c.stream,
                       (const uint8_t*)keys_tiled, (int64_t)g.spi * k3tc::kSubBytes, (const __nv_bfloat16*)a.q, a.P,
                       a.dk, a.top_k, a.scale, a.work, a.counters, a.item_tok, a.work_cap, a.use_slots, a.prim_out,
-                      a.weight_out, a.status, a.keep_mask, (const uint8_t*)a.values, a.vrow_bytes, g);
+                      a.weight_out, a.status, a.selpos, (const uint8_t*)a.values, a.vrow_bytes,
+                      (const uint8_t*)a.hidden0, a.rec_t, a.rec_row, a.rec_w, g);
 }
 
 cudaError_t configure_score_tc_kernel() {

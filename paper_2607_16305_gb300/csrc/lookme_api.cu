@@ -10,6 +10,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <climits>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -130,6 +131,10 @@ struct lookme_table {
     int32_t* counters = nullptr;  // n_work, n_routed, max bucket
     int32_t* sel = nullptr;
     uint8_t* mask = nullptr;
+    int32_t* selpos = nullptr;   // per token: its kept-list slot, or -1
+    int32_t* rec_t = nullptr;    // injection records by kept slot: token id,
+    int32_t* rec_row = nullptr;  // value rows and weights (kRecMaxTopK per slot)
+    float* rec_w = nullptr;
     uint32_t* status = nullptr;   // persistent device status word
     int64_t last_tokens = -1;
     int64_t last_staged_bytes = 0;
@@ -219,6 +224,10 @@ lookme_status ensure_scratch(lookme_table* t, int64_t n, cudaStream_t s) {
     const size_t o_counters = take(4 * sizeof(int32_t));
     const size_t o_sel = take(cap * sizeof(int32_t));
     const size_t o_mask = take(cap);
+    const size_t o_selpos = take(cap * sizeof(int32_t));
+    const size_t o_rec_t = take(cap * sizeof(int32_t));
+    const size_t o_rec_row = take(cap * kRecMaxTopK * sizeof(int32_t));
+    const size_t o_rec_w = take(cap * kRecMaxTopK * sizeof(float));
     void* buf = nullptr;
     if (cudaDeviceSynchronize() != cudaSuccess || cudaMalloc(&buf, off) != cudaSuccess) {
         cudaGetLastError();
@@ -236,6 +245,10 @@ lookme_status ensure_scratch(lookme_table* t, int64_t n, cudaStream_t s) {
     t->counters = reinterpret_cast<int32_t*>(b + o_counters);
     t->sel = reinterpret_cast<int32_t*>(b + o_sel);
     t->mask = reinterpret_cast<uint8_t*>(b + o_mask);
+    t->selpos = reinterpret_cast<int32_t*>(b + o_selpos);
+    t->rec_t = reinterpret_cast<int32_t*>(b + o_rec_t);
+    t->rec_row = reinterpret_cast<int32_t*>(b + o_rec_row);
+    t->rec_w = reinterpret_cast<float*>(b + o_rec_w);
     t->last_tokens = -1;
     if (cudaMemset(buf, 0, off) != cudaSuccess) return cuda_fail(t, cudaGetLastError(), "scratch memset");
     return LOOKME_OK;
@@ -491,7 +504,7 @@ namespace {
 // lookme_lookup; with gate the bucketing kernel also computes the injection gate.
 lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32_t top_k, int32_t* scene_out,
                           int32_t* prim_out, float* weight_out, float* qnorm_out, lookme_stream stream,
-                          const GateSpec* gate) {
+                          const GateSpec* gate, const void* hidden0 = nullptr, bool records = false) {
     lookme_status st = check_table(t);
     if (st != LOOKME_OK) return st;
     const lookme_table_desc& d = t->d;
@@ -565,10 +578,16 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
     a.weight_out = weight_out;
     a.status = t->status;
     // With the gate decided beside the bucketing, level 2 prefetches the kept
-    // tokens' value rows (HBM-resident tables).
-    a.keep_mask = (gate && d.residency == LOOKME_RES_DEVICE) ? gate->mask : nullptr;
+    // tokens' value rows (HBM-resident tables) and, with records, writes each
+    // kept token's injection record at its slot.
+    const bool gated = gate && gate->selpos && d.residency == LOOKME_RES_DEVICE;
+    a.selpos = gated ? gate->selpos : nullptr;
     a.values = t->values;
     a.vrow_bytes = d.d_value * (int64_t)t->esz;
+    a.hidden0 = gated ? hidden0 : nullptr;
+    a.rec_t = gated && records ? t->rec_t : nullptr;
+    a.rec_row = gated && records ? t->rec_row : nullptr;
+    a.rec_w = gated && records ? t->rec_w : nullptr;
     st = launch(t, s, KID_SCORE,
                 [&] { return t->tc_score ? launch_score_tc(ctx, a.keys, a) : launch_score(ctx, a); });
     if (st != LOOKME_OK) return st;
@@ -714,6 +733,7 @@ lookme_status lookme_lookup_inject(lookme_table* t, const void* queries, int64_t
     gs.priority = priority ? priority : t->qnorm;
     gs.mask = mask_out ? mask_out : t->mask;
     gs.sel = t->sel;
+    gs.selpos = t->selpos;
     int64_t base = 0;
     for (int i = 0; i < plan.n_seg; ++i) {
         gs.off[i] = plan.off[i];
@@ -721,12 +741,22 @@ lookme_status lookme_lookup_inject(lookme_table* t, const void* queries, int64_t
         base += (int64_t)std::floor((double)(plan.off[i + 1] - plan.off[i]) * keep_ratio);
     }
     gs.off[plan.n_seg] = plan.off[plan.n_seg];
-    st = lookup_impl(t, queries, N, top_k, scene_out, prim_out, weight_out, nullptr, stream, &gs);
+    // The tcgen05 level-2 kernel writes each kept token's injection record
+    // (token, value rows, weights) at its slot, and the injection reads them
+    // in one round trip.
+    const lookme_table_desc& d = t->d;
+    const bool records = t->tc_score && d.residency == LOOKME_RES_DEVICE && top_k <= kRecMaxTopK &&
+                         d.n_scenes * d.n_prims < (int64_t)INT32_MAX;
+    st = lookup_impl(t, queries, N, top_k, scene_out, prim_out, weight_out, nullptr, stream, &gs, hidden[0],
+                     records);
     if (st != LOOKME_OK) return st;
     if (plan.n_sel == 0) return LOOKME_OK;
     LaunchCtx ctx{s, t->num_sms};
     const InjectArgs a =
         inject_args(t, scene_out, prim_out, weight_out, N, top_k, hidden, n_layers, t->sel, plan.n_sel);
+    if (records)
+        return launch(t, s, KID_INJECT,
+                      [&] { return launch_inject_records(ctx, a, t->rec_t, t->rec_row, t->rec_w); });
     return launch(t, s, KID_INJECT, [&] { return launch_inject(ctx, a); });
 }
 

@@ -8,6 +8,13 @@
 namespace lookme {
 namespace k3 {
 
+// What a lane holds after a top-k: lane j < top_k the j-th selected primitive
+// and its softmax weight, other lanes p = -1.
+struct TopkLane {
+    int p;
+    float w;
+};
+
 // Inverse of orderable(): the float whose order key is u.
 __device__ __forceinline__ float from_orderable(uint32_t u) {
     return __uint_as_float((u & 0x80000000u) ? (u & 0x7FFFFFFFu) : ~u);
@@ -17,7 +24,7 @@ __device__ __forceinline__ float from_orderable(uint32_t u) {
 // index on ties) and the
 // softmax over the selected logits; writes prim/weight of token t (nothing
 // when prim_out is null).
-__device__ __forceinline__ int topk_token(const float* z, int64_t P, int top_k, int lane, int64_t t,
+__device__ __forceinline__ TopkLane topk_token(const float* z, int64_t P, int top_k, int lane, int64_t t,
                                            int32_t* prim_out, float* weight_out, int zs = 1) {
     // Each lane keeps the best untaken element of its slice p = lane + 32 i.
     uint64_t taken = 0ull;
@@ -74,13 +81,13 @@ __device__ __forceinline__ int topk_token(const float* z, int64_t P, int top_k, 
             weight_out[t * top_k + j] = e[h] / sum;
         }
     }
-    return lane < top_k ? my_p[0] : -1;
+    return lane < top_k ? TopkLane{my_p[0], e[0] / sum} : TopkLane{-1, 0.f};
 }
 // Register-resident variant for N_p <= 32 * PPL: each lane holds the order
 // keys of its elements p = 32 i + lane, so a round is an unrolled scan of
 // PPL registers plus two warp reductions.  Same result as topk_token.
 template <int PPL>
-__device__ __forceinline__ int topk_token_regs(const float* z, int64_t P, int top_k, int lane, int64_t t,
+__device__ __forceinline__ TopkLane topk_token_regs(const float* z, int64_t P, int top_k, int lane, int64_t t,
                                                 int32_t* prim_out, float* weight_out, int zs = 1) {
     uint32_t key[PPL];
 #pragma unroll
@@ -134,7 +141,7 @@ __device__ __forceinline__ int topk_token_regs(const float* z, int64_t P, int to
             weight_out[t * top_k + j] = e[h] / sum;
         }
     }
-    return lane < top_k ? my_p[0] : -1;
+    return lane < top_k ? TopkLane{my_p[0], e[0] / sum} : TopkLane{-1, 0.f};
 }
 
 // Sorted-list variant for top_k <= L (L = 8 or 16), N_p <= 32 * PPL.  An
@@ -188,7 +195,7 @@ __device__ __forceinline__ void merge_top_desc(uint64_t (&a)[L], const uint64_t 
 }
 
 template <int PPL, int L>
-__device__ __forceinline__ int topk_token_pop(const float* z, int64_t P, int top_k, int lane, int64_t t,
+__device__ __forceinline__ TopkLane topk_token_pop(const float* z, int64_t P, int top_k, int lane, int64_t t,
                                                int32_t* prim_out, float* weight_out, int zs = 1) {
     constexpr int G = (PPL + L - 1) / L;  // groups of L elements per lane
     uint64_t a[L];
@@ -237,11 +244,11 @@ __device__ __forceinline__ int topk_token_pop(const float* z, int64_t P, int top
         prim_out[t * top_k + lane] = (int32_t)my_p;
         weight_out[t * top_k + lane] = e / sum;
     }
-    return lane < top_k ? (int)my_p : -1;
+    return lane < top_k ? TopkLane{(int)my_p, e / sum} : TopkLane{-1, 0.f};
 }
 
 // Top-k of one token, picking the register-resident variant when N_p allows.
-__device__ __forceinline__ int topk_any(const float* z, int64_t P, int top_k, int lane, int64_t t,
+__device__ __forceinline__ TopkLane topk_any(const float* z, int64_t P, int top_k, int lane, int64_t t,
                                          int32_t* prim_out, float* weight_out, int zs = 1) {
     if (top_k <= 8) {
         if (P <= 64) return topk_token_pop<2, 8>(z, P, top_k, lane, t, prim_out, weight_out, zs);
