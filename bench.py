@@ -148,6 +148,23 @@ def algorithmic_bytes(w, n_routed, n_sel):
             "step": score + route + inject + N * 4 * 3 - N * dk * e}  # queries are read once per step
 
 
+def aggregate_ranks(total_ms, e2e_ms, ws, n_tokens, steps, device):
+    """Whole-job numbers over ws replicas (weak scaling): the slowest rank's
+    timed totals, and value = tokens all ranks processed / that time.  With
+    ws > 1 the process group must be initialised (NCCL on the GPUs; any backend
+    whose tensors live on `device`)."""
+    if ws > 1:
+        import torch
+        import torch.distributed as dist
+
+        tt = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms, e2e_ms = tt.tolist()
+    value = ws * n_tokens * steps / (total_ms / 1e3)
+    e2e_value = ws * n_tokens * steps / (e2e_ms / 1e3)
+    return total_ms, e2e_ms, value, e2e_value
+
+
 def run_lookme(args, w, ws, rank, local):
     import torch
 
@@ -294,18 +311,11 @@ def run_lookme(args, w, ws, rank, local):
     clocks = sampler.stop()
     assert t.device_status() == 0, "a device-side wait timed out"
 
-    if ws > 1:
-        import torch.distributed as dist
-
-        tt = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms, e2e_ms = tt.tolist()
+    total_ms, e2e_ms, value, e2e_value = aggregate_ranks(total_ms, e2e_ms, ws, N, args.steps, dev)
 
     h2d = q.numel() * q.element_size() + sum(h.numel() * h.element_size() for h in hidden)
     d2h = sum(h.numel() * h.element_size() for h in hidden)
     ms_per_step = total_ms / args.steps
-    value = ws * N * args.steps / (total_ms / 1e3)
-    e2e_value = ws * N * args.steps / (e2e_ms / 1e3)
 
     peaks, peak_kind = load_peaks()
     hbm = float(peaks["hbm_gbs"])
