@@ -15,9 +15,10 @@
 //   counters[0..3] number of work items, of routed scenes, largest bucket;
 //                  [3] is reset to 0 for the level-2 kernel's work taking
 //
-// With a gate, CTAs 1.. compute the injection gate meanwhile, eight tokens
-// per CTA (one per warp; a light load per SM so they finish within the
-// bucketing): rank_t = #{ j in segment : pi_j > pi_t, or pi_j == pi_t and
+// With a gate, CTAs 1.. compute the injection gate meanwhile, one token per
+// warp and 8 to 32 tokens per CTA (few per CTA when the call is small, so the
+// ranks spread over many SMs and finish within the bucketing; up to all 32
+// warps when there are many): rank_t = #{ j in segment : pi_j > pi_t, or pi_j == pi_t and
 // j < t }, kept iff rank_t < r, the kept ones listed at sel[sel_base + rank_t]
 // (and, optionally, that slot recorded per token in selpos, -1 if not kept).
 // Each CTA stages the priorities its tokens' segments span in shared memory
@@ -33,7 +34,7 @@ namespace lookme {
 
 namespace {
 constexpr int kThreads = 1024;
-constexpr int kGateTokens = 8;     // tokens per gate CTA
+constexpr int kGateMaxTokens = kThreads / 32;  // tokens per gate CTA: at most one per warp
 constexpr int kGateStage = 32768;  // bytes of priorities a gate CTA stages
 
 __device__ __forceinline__ int segment_index(const GateSpec& gs, int64_t t) {
@@ -46,9 +47,9 @@ __device__ __forceinline__ int segment_index(const GateSpec& gs, int64_t t) {
     return lo;
 }
 
-__device__ void gate_block(const GateSpec& gs, float* buf, int cap) {
+__device__ void gate_block(const GateSpec& gs, float* buf, int cap, int tpc) {
     const int tid = threadIdx.x, warp = tid / 32, lane = tid % 32;
-    const int64_t tb = (int64_t)(blockIdx.x - 1) * kGateTokens, te = min(gs.N, tb + kGateTokens);
+    const int64_t tb = (int64_t)(blockIdx.x - 1) * tpc, te = min(gs.N, tb + tpc);
     if (tb >= te) return;  // uniform for the CTA
     const int64_t rb = gs.off[segment_index(gs, tb)], re = gs.off[segment_index(gs, te - 1) + 1];
     const bool staged = re - rb <= cap;  // uniform for the CTA
@@ -57,7 +58,7 @@ __device__ void gate_block(const GateSpec& gs, float* buf, int cap) {
         __syncthreads();
     }
     const int64_t t = tb + warp;
-    if (warp >= kGateTokens || t >= te) return;
+    if (warp >= tpc || t >= te) return;
     const int sg = segment_index(gs, t);
     const int64_t b = gs.off[sg], len = gs.off[sg + 1] - b;
     const int64_t r = (int64_t)floor((double)len * gs.keep_ratio);
@@ -135,14 +136,14 @@ __device__ void block_exclusive_scan2(int2 v, int2& excl, int2& total, int2* war
 __global__ void __launch_bounds__(kThreads, 1)
     k2_bucket(unsigned long long* best, int64_t N, int S, int32_t* __restrict__ scene_out,
               int32_t* __restrict__ item_tok, WorkItem* __restrict__ work, int32_t* __restrict__ routed,
-              int32_t* __restrict__ counters, const __grid_constant__ GateSpec gate, int smem_bytes) {
+              int32_t* __restrict__ counters, const __grid_constant__ GateSpec gate, int smem_bytes, int gate_tpc) {
     extern __shared__ int cnt[];  // CTA 0: [S] counts, then running item_tok positions; gate CTAs: priorities
     __shared__ int2 warp_buf[33];
     __shared__ int max_bucket;
     pdl_trigger();
     pdl_wait();
     if (blockIdx.x > 0) {
-        gate_block(gate, reinterpret_cast<float*>(cnt), smem_bytes / 4);
+        gate_block(gate, reinterpret_cast<float*>(cnt), smem_bytes / 4, gate_tpc);
         return;
     }
     const int tid = threadIdx.x;
@@ -244,10 +245,13 @@ cudaError_t launch_bucket(const LaunchCtx& c, unsigned long long* best, int64_t 
     } else {
         memset(&gs, 0, sizeof(gs));
     }
-    const int gate_ctas = gate ? (int)((N + kGateTokens - 1) / kGateTokens) : 0;
+    // Tokens per gate CTA: about two gate CTAs per SM, 8 to 32 tokens each.
+    const int64_t want = (N + 2 * (int64_t)c.num_sms - 1) / (2 * (int64_t)c.num_sms);
+    const int tpc = (int)std::min<int64_t>(kGateMaxTokens, std::max<int64_t>(8, want));
+    const int gate_ctas = gate ? (int)((N + tpc - 1) / tpc) : 0;
     const int smem = (int)std::max<int64_t>(S * (int64_t)sizeof(int), gate ? kGateStage : 0);
     return launch_pdl(k2_bucket, dim3(1 + gate_ctas), dim3(kThreads), (size_t)smem, c.stream, best, N, (int)S,
-                      scene_out, item_tok, work, routed, counters, gs, smem);
+                      scene_out, item_tok, work, routed, counters, gs, smem, tpc);
 }
 
 cudaError_t configure_bucket_kernel() {
