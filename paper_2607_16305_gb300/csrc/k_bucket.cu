@@ -150,31 +150,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = tid; s < S; s += kThreads) cnt[s] = 0;
     if (tid == 0) max_bucket = 0;
     __syncthreads();
-    // The scenes of a thread's first kCache tokens stay in registers for the
-    // second sweep (no second read of the keys).
-    constexpr int kCache = 4;
-    int32_t sc[kCache];
-    {
-        unsigned long long key[kCache];
+    // Both sweeps over the tokens issue kB keys per thread before using any
+    // (one round trip per batch, not per token); the scenes of a thread's
+    // first batch stay in registers for the second sweep.
+    constexpr int kB = 8;
+    int32_t sc[kB];
+    for (int64_t t0 = tid; t0 < N; t0 += (int64_t)kB * kThreads) {
+        unsigned long long key[kB];
 #pragma unroll
-        for (int u = 0; u < kCache; ++u) {
-            const int64_t t = tid + (int64_t)u * kThreads;
+        for (int u = 0; u < kB; ++u) {
+            const int64_t t = t0 + (int64_t)u * kThreads;
             key[u] = t < N ? best[t] : 0ull;
         }
 #pragma unroll
-        for (int u = 0; u < kCache; ++u) {
-            const int64_t t = tid + (int64_t)u * kThreads;
-            sc[u] = unpack_scene(key[u], S);
+        for (int u = 0; u < kB; ++u) {
+            const int64_t t = t0 + (int64_t)u * kThreads;
+            const int32_t s = unpack_scene(key[u], S);
+            if (t0 == tid) sc[u] = s;
             if (t < N) {
-                scene_out[t] = sc[u];
-                atomicAdd(&cnt[sc[u]], 1);
+                scene_out[t] = s;
+                atomicAdd(&cnt[s], 1);
             }
         }
-    }
-    for (int64_t t = tid + (int64_t)kCache * kThreads; t < N; t += kThreads) {
-        const int32_t s = unpack_scene(best[t], S);
-        scene_out[t] = s;
-        atomicAdd(&cnt[s], 1);
     }
     __syncthreads();
 
@@ -219,20 +216,30 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     // A scene's k-th token lands in its item k / 8, lane k % 8; the keys are
     // cleared for the next call's argmax.
+    for (int64_t t0 = tid; t0 < N; t0 += (int64_t)kB * kThreads) {
+        int32_t s[kB];
+        if (t0 == tid) {
 #pragma unroll
-    for (int u = 0; u < kCache; ++u) {
-        const int64_t t = tid + (int64_t)u * kThreads;
-        if (t < N) {
-            best[t] = 0ull;
-            const int pos = atomicAdd(&cnt[sc[u]], 1);
-            item_tok[pos] = (int32_t)t;
+            for (int u = 0; u < kB; ++u) s[u] = sc[u];
+        } else {
+            unsigned long long key[kB];
+#pragma unroll
+            for (int u = 0; u < kB; ++u) {
+                const int64_t t = t0 + (int64_t)u * kThreads;
+                key[u] = t < N ? best[t] : 0ull;
+            }
+#pragma unroll
+            for (int u = 0; u < kB; ++u) s[u] = unpack_scene(key[u], S);
         }
-    }
-    for (int64_t t = tid + (int64_t)kCache * kThreads; t < N; t += kThreads) {
-        const int32_t s = unpack_scene(best[t], S);
-        best[t] = 0ull;
-        const int pos = atomicAdd(&cnt[s], 1);
-        item_tok[pos] = (int32_t)t;
+#pragma unroll
+        for (int u = 0; u < kB; ++u) {
+            const int64_t t = t0 + (int64_t)u * kThreads;
+            if (t < N) {
+                best[t] = 0ull;
+                const int pos = atomicAdd(&cnt[s[u]], 1);
+                item_tok[pos] = (int32_t)t;
+            }
+        }
     }
 }
 

@@ -152,13 +152,16 @@ cudaError_t launch_route_simt(const LaunchCtx& c, int dtype, const void* q, cons
 //   warp 1      MMA issuer (one thread): D[buf] = Q_tile * C_tile^T in TMEM,
 //               two accumulator buffers so the epilogue of tile i overlaps
 //               the MMAs of tile i+1
-//   warps 2..5  epilogue: each thread owns one token row (one TMEM lane),
-//               reads the BN scores of its row, keeps the best (score, scene)
-//               and finally merges it with one atomicMax per row
+//   warps 2..9  epilogue: two warps per TMEM lane quarter, each thread one
+//               token row (one TMEM lane) and half of the tile's BN columns;
+//               it keeps the best (score, scene) of what it read, a strict
+//               float compare in increasing scene order (ties keep the lowest
+//               scene), and merges it with one atomicMax per row and half
 namespace k1tc {
 constexpr int BM = 128;
 constexpr int BK = 64;              // bf16 elements per 128-byte swizzled row
-constexpr int kThreads = 192;
+constexpr int kEpiWarps = 8;  // two per TMEM lane quarter, each half of a tile's columns
+constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 
 __host__ __device__ constexpr int smem_bytes(int BN, int STAGES, int nkb) {
@@ -166,16 +169,16 @@ __host__ __device__ constexpr int smem_bytes(int BN, int STAGES, int nkb) {
            4 * BN * 4 /*per-tile scene constants, double-buffered*/;
 }
 
-// Named barrier 1 over the four epilogue warps, returning the OR of `v`.
+// Named barrier 1 over the epilogue warps, returning the OR of `v`.
 __device__ __forceinline__ bool epi_sync_or(bool v) {
     uint32_t r;
     asm volatile(
         "{\n\t.reg .pred p, q;\n\t"
         "setp.ne.u32 p, %1, 0;\n\t"
-        "bar.red.or.pred q, 1, 128, p;\n\t"
+        "bar.red.or.pred q, 1, %2, p;\n\t"
         "selp.u32 %0, 1, 0, q;\n\t}"
         : "=r"(r)
-        : "r"((uint32_t)v)
+        : "r"((uint32_t)v), "n"(32 * kEpiWarps)
         : "memory");
     return r != 0;
 }
@@ -221,7 +224,7 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
         ptx::mbar_init(a_full, 1);
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(&t_full[i], 1);
-            ptx::mbar_init(&t_empty[i], 4);  // one arrival per epilogue warp
+            ptx::mbar_init(&t_empty[i], kEpiWarps);  // one arrival per epilogue warp
         }
         ptx::mbar_init(drain, 1);
         *abort = 0;
@@ -300,15 +303,19 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
             ptx::mbar_wait_drain(drain, 0, kTimeoutNs);
         }
     } else {
-        // Epilogue warps 2..5 own TMEM lane quarters (warp % 4) * 32 .. + 31.
+        // Epilogue warps 2..9: warp w owns TMEM lane quarter (w % 4) * 32 .. + 31
+        // and column half (w - 2) / 4 of every tile.
         const int quarter = warp & 3;
+        const int half = (warp - 2) / 4;
+        constexpr int HC = BN / 2;  // columns per warp and tile
         const int64_t row = (int64_t)m_tile * BM + quarter * 32 + lane;
         // ||q_row||_2 from the token tile in shared memory: every 16-byte chunk
         // of the row is read once (lane-rotated to avoid bank conflicts; the
         // swizzle only permutes chunks within the row, and zero-filled columns
-        // past d_k add nothing).
+        // past d_k add nothing).  Both warps of a quarter need it with a bias;
+        // the first half's warp stores it.
         float inv_q = 1.f;
-        if (blockIdx.y == 0 || bias) {
+        if ((blockIdx.y == 0 && half == 0) || bias) {
             const bool ready = ptx::mbar_wait(a_full, 0, abort, kTimeoutNs);
             float ss = 0.f;
             if (ready) {
@@ -325,31 +332,34 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
                 }
             }
             const float n = sqrtf(ss);
-            if (blockIdx.y == 0 && row < N && ready) {
+            if (blockIdx.y == 0 && half == 0 && row < N && ready) {
                 qnorm[row] = n;
                 if (qnorm_out) qnorm_out[row] = n;
             }
             if (bias) inv_q = n > 0.f ? 1.f / n : 0.f;
         }
-        // Scene constants of the next tile are loaded while this one is scored.
-        const int et = threadIdx.x - 64;  // 0..127
-        constexpr int PER = (BN + 127) / 128;
+        // Scene constants of the next tile are loaded while this one is scored;
+        // columns past S get NaN, which no score compare ever selects.
+        const int et = threadIdx.x - 64;  // 0 .. 32 kEpiWarps - 1
+        constexpr int ET = 32 * kEpiWarps;
+        constexpr int PER = (BN + ET - 1) / ET;
+        const float nan = __int_as_float(0x7fc00000);
         float ic_next[PER], b_next[PER];
         auto load_consts = [&](int nt) {
 #pragma unroll
             for (int u = 0; u < PER; ++u) {
-                const int64_t s = (int64_t)nt * BN + et + u * 128;
-                const bool in = et + u * 128 < BN && s < S;
-                ic_next[u] = in ? __ldg(inv_cnorm + s) : 0.f;
+                const int64_t s = (int64_t)nt * BN + et + u * ET;
+                const bool in = et + u * ET < BN && s < S;
+                ic_next[u] = in ? __ldg(inv_cnorm + s) : nan;
                 b_next[u] = (in && bias) ? __ldg(bias + s) : 0.f;
             }
         };
         auto store_consts = [&](int buf) {
 #pragma unroll
             for (int u = 0; u < PER; ++u) {
-                if (et + u * 128 < BN) {
-                    s_ic[buf * BN + et + u * 128] = ic_next[u];
-                    s_bias[buf * BN + et + u * 128] = b_next[u];
+                if (et + u * ET < BN) {
+                    s_ic[buf * BN + et + u * ET] = ic_next[u];
+                    s_bias[buf * BN + et + u * ET] = b_next[u];
                 }
             }
         };
@@ -357,7 +367,8 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
             load_consts(nt0);
             store_consts(0);
         }
-        unsigned long long key = 0ull;
+        float best_v = -INFINITY;
+        int64_t best_s = -1;
         for (int it = 0, nt = nt0; nt < nt1; ++nt, ++it) {
             const int buf = it & 1;
             const uint32_t use = (uint32_t)(it >> 1);
@@ -367,29 +378,39 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
             const bool ready = ptx::mbar_wait(&t_full[buf], use & 1u, abort, kTimeoutNs);
             if (k1tc::epi_sync_or(!__all_sync(0xFFFFFFFFu, ready))) break;
             ptx::tc_fence_after();
-            const int64_t s_base = (int64_t)nt * BN;
-            const float* ic = s_ic + buf * BN;
-            const float* bs = s_bias + buf * BN;
+            const int c0 = half * HC;
+            const float* ic = s_ic + buf * BN + c0;
+            const float* bs = s_bias + buf * BN + c0;
+            // The best column of this tile's half: strict > in increasing column
+            // order keeps the lowest scene among equal scores.
+            float tv = -INFINITY;
+            int tc = -1;
 #pragma unroll 1
-            for (int c = 0; c < BN; c += 32) {
+            for (int c = 0; c < HC; c += 32) {
                 uint32_t r[32];
-                ptx::tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN + c), r);
+                ptx::tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN + c0 + c),
+                                        r);
                 ptx::tmem_wait_ld();
 #pragma unroll
                 for (int j = 0; j < 32; ++j) {
-                    const int64_t s = s_base + c + j;
                     float score = __uint_as_float(r[j]) * ic[c + j];
                     if (bias) score = fmaf(score, inv_q, bs[c + j]);
-                    const unsigned long long k = pack_argmax(score, (uint32_t)s);
-                    if (s < S) key = k > key ? k : key;
+                    if (score > tv) {
+                        tv = score;
+                        tc = c + j;
+                    }
                 }
             }
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&t_empty[buf]);
             if (nt + 1 < nt1) store_consts(buf ^ 1);
+            if (tc >= 0 && tv > best_v) {  // later tiles hold larger scene indices
+                best_v = tv;
+                best_s = (int64_t)nt * BN + c0 + tc;
+            }
         }
-        if (row < N && key && !*abort) atomicMax(&best[row], key);
+        if (row < N && best_s >= 0 && !*abort) atomicMax(&best[row], pack_argmax(best_v, (uint32_t)best_s));
     }
 
     ptx::tc_fence_before();
