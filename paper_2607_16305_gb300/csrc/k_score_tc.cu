@@ -485,13 +485,21 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
                     ptx::tc_fence_after();
                     const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) +
                                            (uint32_t)(buf * (g.tmem_cols >> 1) + c0);
-#pragma unroll 1
-                    for (int h = 0; h < 32 && c0 + h < ncols; h += 16) {
-                        uint32_t r[16];
-                        ptx::tmem_ld_32x32b_x16(taddr + (uint32_t)h, r);
+                    const int64_t p0 = (int64_t)nt * kNTile + c0;
+                    if (c0 + 32 <= ncols) {  // one load and one wait for the warp's 32 columns
+                        uint32_t r[32];
+                        ptx::tmem_ld_32x32b_x32(taddr, r);
                         ptx::tmem_wait_ld();
                         if (lane < nb) {
-                            const int64_t p0 = (int64_t)nt * kNTile + c0 + h;
+#pragma unroll
+                            for (int j = 0; j < 32; ++j)
+                                if (p0 + j < P) zg[(p0 + j) * kZStride + lane] = __uint_as_float(r[j]) * scale;
+                        }
+                    } else {  // 16 columns (N is a multiple of 16)
+                        uint32_t r[16];
+                        ptx::tmem_ld_32x32b_x16(taddr, r);
+                        ptx::tmem_wait_ld();
+                        if (lane < nb) {
 #pragma unroll
                             for (int j = 0; j < 16; ++j)
                                 if (p0 + j < P) zg[(p0 + j) * kZStride + lane] = __uint_as_float(r[j]) * scale;
