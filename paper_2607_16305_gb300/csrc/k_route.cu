@@ -7,6 +7,8 @@
 // into a per-token 64-bit key with atomicMax, so scores never reach HBM.
 #include <cuda.h>
 
+#include <algorithm>
+
 #include "common.cuh"
 #include "sm100.cuh"
 
@@ -146,9 +148,15 @@ cudaError_t launch_route_simt(const LaunchCtx& c, int dtype, const void* q, cons
 }
 
 // ---------------------------------------------------- K1 on tcgen05 (bf16)
-// One CTA = one 128-token tile (MMA M) and a run of BN-scene tiles (MMA N).
-//   warp 0      TMA producer: the token tile once (all of d_k), then the
-//               centroid tiles through a STAGES-deep ring of 64-wide k-blocks
+// Work units are (128-token tile (MMA M), BN-scene tile (MMA N)) pairs in
+// token-tile-major order; CTA b takes the contiguous run of units
+// [b u, (b + 1) u), one CTA per SM, so that every SM gets the same number of
+// tiles whatever the grid of tiles (a run crosses into the next token tile
+// by reloading the token tile once the previous one's MMAs and norm reads
+// are done).
+//   warp 0      TMA producer: each token tile of the run once (all of d_k),
+//               the centroid tiles through a STAGES-deep ring of 64-wide
+//               k-blocks
 //   warp 1      MMA issuer (one thread): D[buf] = Q_tile * C_tile^T in TMEM,
 //               two accumulator buffers so the epilogue of tile i overlaps
 //               the MMAs of tile i+1
@@ -187,7 +195,7 @@ __device__ __forceinline__ bool epi_sync_or(bool v) {
 template <int BN, int STAGES>
 __global__ void __launch_bounds__(k1tc::kThreads, 1)
     k1_route_tc(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_c,
-                int64_t N, int64_t S, int dk, int tiles_per_cta, const float* __restrict__ inv_cnorm,
+                int64_t N, int64_t S, int dk, int units_per_cta, const float* __restrict__ inv_cnorm,
                 const float* __restrict__ bias, float* __restrict__ qnorm, float* __restrict__ qnorm_out,
                 unsigned long long* __restrict__ best, uint32_t* __restrict__ status) {
     using namespace k1tc;
@@ -199,7 +207,8 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
     uint64_t* full = reinterpret_cast<uint64_t*>(sB + STAGES * BN * 128);
     uint64_t* empty = full + STAGES;
     uint64_t* a_full = empty + STAGES;
-    uint64_t* t_full = a_full + 1;   // [2]
+    uint64_t* a_empty = a_full + 1;  // the token tile's MMAs and norm reads are done
+    uint64_t* t_full = a_empty + 1;  // [2]
     uint64_t* t_empty = t_full + 2;  // [2]
     uint64_t* drain = t_empty + 2;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
@@ -209,10 +218,10 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
     float* s_bias = s_ic + 2 * BN;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int m_tile = blockIdx.x;
     const int n_tiles = (int)((S + BN - 1) / BN);
-    const int nt0 = blockIdx.y * tiles_per_cta;
-    const int nt1 = min(n_tiles, nt0 + tiles_per_cta);
+    const int64_t n_units = (int64_t)((N + BM - 1) / BM) * n_tiles;
+    const int64_t u0 = (int64_t)blockIdx.x * units_per_cta;
+    const int64_t u1 = min(n_units, u0 + units_per_cta);
 
     if (threadIdx.x == 0) {
         ptx::prefetch_tmap(&tmap_q);
@@ -222,6 +231,7 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
             ptx::mbar_init(&empty[i], 1);
         }
         ptx::mbar_init(a_full, 1);
+        ptx::mbar_init(a_empty, 1 + kEpiWarps);  // the MMA issuer's commit and each epilogue warp
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(&t_full[i], 1);
             ptx::mbar_init(&t_empty[i], kEpiWarps);  // one arrival per epilogue warp
@@ -241,16 +251,26 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
     const uint32_t tmem_base = *tmem_slot;
 
     if (warp == 0) {
-        if (lane == 0 && nt0 < nt1) {
-            ptx::mbar_arrive_expect_tx(a_full, (uint32_t)(nkb * BM * 128));
-            for (int kb = 0; kb < nkb; ++kb)
-                ptx::tma_load_2d(sA + kb * BM * 128, &tmap_q, kb * BK, m_tile * BM, a_full);
+        if (lane == 0 && u0 < u1) {
             int stage = 0;
             uint32_t phase = 0;
             uint32_t issued = 0;      // bit i: ring slot i has been written at least once
             uint32_t last_par = 0;    // bit i: parity of slot i's most recent fill
+            int seg = -1;             // token tiles loaded so far - 1
+            int64_t m_cur = -1;
             bool ok = true;
-            for (int nt = nt0; nt < nt1 && ok; ++nt) {
+            for (int64_t u = u0; u < u1 && ok; ++u) {
+                const int64_t m = u / n_tiles;
+                const int nt = (int)(u - m * n_tiles);
+                if (m != m_cur) {
+                    // The previous token tile's MMAs and norm reads are done before it is overwritten.
+                    if (seg >= 0 && !(ok = ptx::mbar_wait(a_empty, (uint32_t)(seg & 1), abort, kTimeoutNs))) break;
+                    ++seg;
+                    m_cur = m;
+                    ptx::mbar_arrive_expect_tx(a_full, (uint32_t)(nkb * BM * 128));
+                    for (int kb = 0; kb < nkb; ++kb)
+                        ptx::tma_load_2d(sA + kb * BM * 128, &tmap_q, kb * BK, (int32_t)(m * BM), a_full);
+                }
                 for (int kb = 0; kb < nkb; ++kb) {
                     if (!(ok = ptx::mbar_wait(&empty[stage], phase ^ 1u, abort, kTimeoutNs))) break;
                     ptx::mbar_arrive_expect_tx(&full[stage], (uint32_t)(BN * 128));
@@ -264,18 +284,28 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
                 }
             }
             // Every copy this thread issued must have landed before the CTA exits.
-            ptx::mbar_wait_drain(a_full, 0, kTimeoutNs);
+            if (seg >= 0) ptx::mbar_wait_drain(a_full, (uint32_t)(seg & 1), kTimeoutNs);
             for (int i = 0; i < STAGES; ++i)
                 if (issued & (1u << i)) ptx::mbar_wait_drain(&full[i], (last_par >> i) & 1u, kTimeoutNs);
         }
     } else if (warp == 1) {
-        if (lane == 0 && nt0 < nt1) {
+        if (lane == 0 && u0 < u1) {
             constexpr uint32_t idesc = ptx::idesc_bf16_f32<BM, BN>();
-            bool ok = ptx::mbar_wait(a_full, 0, abort, kTimeoutNs);
+            bool ok = true;
             int stage = 0;
             uint32_t phase = 0;
-            for (int it = 0, nt = nt0; nt < nt1 && ok; ++nt, ++it) {
-                const int buf = it & 1;
+            int seg = -1;
+            int64_t m_cur = -1;
+            for (int64_t u = u0, it = 0; u < u1 && ok; ++u, ++it) {
+                const int64_t m = u / n_tiles;
+                if (m != m_cur) {
+                    // The previous token tile is free once the MMAs issued so far complete.
+                    if (seg >= 0) ptx::mma_commit(a_empty);
+                    ++seg;
+                    m_cur = m;
+                    if (!(ok = ptx::mbar_wait(a_full, (uint32_t)(seg & 1), abort, kTimeoutNs))) break;
+                }
+                const int buf = (int)(it & 1);
                 const uint32_t use = (uint32_t)(it >> 1);
                 if (!(ok = ptx::mbar_wait(&t_empty[buf], (use & 1u) ^ 1u, abort, kTimeoutNs))) break;
                 ptx::tc_fence_after();
@@ -308,36 +338,6 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
         const int quarter = warp & 3;
         const int half = (warp - 2) / 4;
         constexpr int HC = BN / 2;  // columns per warp and tile
-        const int64_t row = (int64_t)m_tile * BM + quarter * 32 + lane;
-        // ||q_row||_2 from the token tile in shared memory: every 16-byte chunk
-        // of the row is read once (lane-rotated to avoid bank conflicts; the
-        // swizzle only permutes chunks within the row, and zero-filled columns
-        // past d_k add nothing).  Both warps of a quarter need it with a bias;
-        // the first half's warp stores it.
-        float inv_q = 1.f;
-        if ((blockIdx.y == 0 && half == 0) || bias) {
-            const bool ready = ptx::mbar_wait(a_full, 0, abort, kTimeoutNs);
-            float ss = 0.f;
-            if (ready) {
-                const int r = quarter * 32 + lane;
-                for (int kb = 0; kb < nkb; ++kb) {
-#pragma unroll
-                    for (int c = 0; c < 8; ++c) {
-                        float f[8];
-                        Vec16<__nv_bfloat16>::unpack(
-                            *reinterpret_cast<const uint4*>(sA + kb * BM * 128 + r * 128 + (((c + lane) & 7) * 16)), f);
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) ss = fmaf(f[i], f[i], ss);
-                    }
-                }
-            }
-            const float n = sqrtf(ss);
-            if (blockIdx.y == 0 && half == 0 && row < N && ready) {
-                qnorm[row] = n;
-                if (qnorm_out) qnorm_out[row] = n;
-            }
-            if (bias) inv_q = n > 0.f ? 1.f / n : 0.f;
-        }
         // Scene constants of the next tile are loaded while this one is scored;
         // columns past S get NaN, which no score compare ever selects.
         const int et = threadIdx.x - 64;  // 0 .. 32 kEpiWarps - 1
@@ -363,16 +363,62 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
                 }
             }
         };
-        if (nt0 < nt1) {
-            load_consts(nt0);
+        if (u0 < u1) {
+            load_consts((int)(u0 % n_tiles));
             store_consts(0);
         }
         float best_v = -INFINITY;
-        int64_t best_s = -1;
-        for (int it = 0, nt = nt0; nt < nt1; ++nt, ++it) {
-            const int buf = it & 1;
+        int64_t best_s = -1, row = -1;
+        float inv_q = 1.f;
+        int seg = -1;
+        int64_t m_cur = -1;
+        for (int64_t u = u0, it = 0; u < u1; ++u, ++it) {
+            const int64_t m = u / n_tiles;
+            const int nt = (int)(u - m * n_tiles);
+            const int buf = (int)(it & 1);
             const uint32_t use = (uint32_t)(it >> 1);
-            if (nt + 1 < nt1) load_consts(nt + 1);
+            if (u + 1 < u1) load_consts((int)((u + 1) % n_tiles));
+            if (m != m_cur) {
+                // The finished token tile's rows, then the new tile's norms: ||q_row||_2
+                // from the token tile in shared memory, every 16-byte chunk of the
+                // row read once (lane-rotated to avoid bank conflicts; the swizzle
+                // only permutes chunks within the row, and zero-filled columns past
+                // d_k add nothing).  The unit with scene tile 0 (one CTA) stores it;
+                // with a bias every warp needs it.
+                if (row >= 0 && row < N && best_s >= 0 && !*abort)
+                    atomicMax(&best[row], pack_argmax(best_v, (uint32_t)best_s));
+                best_v = -INFINITY;
+                best_s = -1;
+                ++seg;
+                m_cur = m;
+                row = m * BM + quarter * 32 + lane;
+                const bool ready = ptx::mbar_wait(a_full, (uint32_t)(seg & 1), abort, kTimeoutNs);
+                const bool store = nt == 0 && half == 0;
+                if (ready && (store || bias)) {
+                    float ss = 0.f;
+                    const int r = quarter * 32 + lane;
+                    for (int kb = 0; kb < nkb; ++kb) {
+#pragma unroll
+                        for (int c = 0; c < 8; ++c) {
+                            float f[8];
+                            Vec16<__nv_bfloat16>::unpack(
+                                *reinterpret_cast<const uint4*>(sA + kb * BM * 128 + r * 128 + (((c + lane) & 7) * 16)),
+                                f);
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) ss = fmaf(f[i], f[i], ss);
+                        }
+                    }
+                    const float n = sqrtf(ss);
+                    if (store && row < N) {
+                        qnorm[row] = n;
+                        if (qnorm_out) qnorm_out[row] = n;
+                    }
+                    if (bias) inv_q = n > 0.f ? 1.f / n : 0.f;
+                }
+                // This warp is done with the token tile.
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(a_empty);
+            }
             // Warp-uniform wait (tcgen05.ld below must be executed by the whole
             // warp); the barrier also publishes this tile's constants.
             const bool ready = ptx::mbar_wait(&t_full[buf], use & 1u, abort, kTimeoutNs);
@@ -404,13 +450,13 @@ __global__ void __launch_bounds__(k1tc::kThreads, 1)
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&t_empty[buf]);
-            if (nt + 1 < nt1) store_consts(buf ^ 1);
-            if (tc >= 0 && tv > best_v) {  // later tiles hold larger scene indices
+            if (u + 1 < u1) store_consts(buf ^ 1);
+            if (tc >= 0 && tv > best_v) {  // later tiles of a token tile hold larger scene indices
                 best_v = tv;
                 best_s = (int64_t)nt * BN + c0 + tc;
             }
         }
-        if (row < N && best_s >= 0 && !*abort) atomicMax(&best[row], pack_argmax(best_v, (uint32_t)best_s));
+        if (row >= 0 && row < N && best_s >= 0 && !*abort) atomicMax(&best[row], pack_argmax(best_v, (uint32_t)best_s));
     }
 
     ptx::tc_fence_before();
@@ -435,19 +481,18 @@ static cudaError_t launch_route_tc_t(const LaunchCtx& c, const void* tmap_q, con
     // (max_resident + 1) CTAs, each with 1 KB of system shared memory, must not fit in 228 KB.
     const int floor_bytes = (228 * 1024) / (max_resident + 1) - 1024 + 1;
     if (smem < floor_bytes) smem = floor_bytes;
-    const int m_tiles = (int)((N + BM - 1) / BM);
-    const int n_tiles = (int)((S + BN - 1) / BN);
-    // Split the scene tiles so that the grid covers the SMs about once.
-    int splits = (c.num_sms + m_tiles - 1) / m_tiles;
-    if (splits > n_tiles) splits = n_tiles;
-    if (splits < 1) splits = 1;
-    const int per = (n_tiles + splits - 1) / splits;
-    splits = (n_tiles + per - 1) / per;
+    const int64_t m_tiles = (N + BM - 1) / BM;
+    const int64_t n_tiles = (S + BN - 1) / BN;
+    // One CTA per SM, each a contiguous run of (token tile, scene tile) units.
+    const int64_t units = m_tiles * n_tiles;
+    int64_t grid = std::min<int64_t>(units, c.num_sms);
+    const int64_t per = (units + grid - 1) / grid;
+    grid = (units + per - 1) / per;
     CUtensorMap mq, mc;
     memcpy(&mq, tmap_q, sizeof(CUtensorMap));
     memcpy(&mc, tmap_c, sizeof(CUtensorMap));
-    return launch_pdl(k1_route_tc<BN, STAGES>, dim3(m_tiles, splits), dim3(kThreads), (size_t)smem, c.stream, mq, mc,
-                      N, S, dk, per, inv_cnorm, bias, qnorm, qnorm_out, best, status);
+    return launch_pdl(k1_route_tc<BN, STAGES>, dim3((unsigned)grid), dim3(kThreads), (size_t)smem, c.stream, mq, mc,
+                      N, S, dk, (int)per, inv_cnorm, bias, qnorm, qnorm_out, best, status);
 }
 
 cudaError_t launch_route_tc(const LaunchCtx& c, const void* tmap_q, const void* const tmap_c[3], int64_t N,
