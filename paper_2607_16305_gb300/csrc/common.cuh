@@ -27,6 +27,9 @@ enum KernelId : int32_t {
     KID_ROUTE_DECODE = 10,  // argmax key -> scene id (allocation-free routing)
     KID_SELECT_INJECT = 11, // K5 + K4 fused for short segments
     KID_TILE_KEYS = 12,  // load-time: keys into the tcgen05 level-2 tile layout
+    KID_BUCKET_COUNT = 13,    // K2 for large calls: per-scene counts (+ gate CTAs)
+    KID_BUCKET_SCAN = 14,     // K2 for large calls: work list from the counts
+    KID_BUCKET_SCATTER = 15,  // K2 for large calls: token ids into their items
     KID_COUNT
 };
 
@@ -151,6 +154,18 @@ struct GateSpec;
 cudaError_t launch_bucket(const LaunchCtx& c, unsigned long long* best, int64_t N, int64_t S,
                           int32_t* scene_out, int32_t* item_tok, WorkItem* work, int32_t* routed, int32_t* counters,
                           const GateSpec* gate = nullptr);
+// The same result for calls of more than kBucketOneCtaTokens tokens, in three
+// launches over all SMs: per-scene counts (global, warp-aggregated atomics;
+// the gate CTAs ride along), the work list from the counts (one CTA; it also
+// zeroes the counts for the next call), and the token ids into their items.
+// cnt [S] must be zero on entry; pos [S] is scratch.
+constexpr int64_t kBucketOneCtaTokens = 8192;
+cudaError_t launch_bucket_count(const LaunchCtx& c, unsigned long long* best, int64_t N, int64_t S,
+                                int32_t* scene_out, int32_t* cnt, const GateSpec* gate);
+cudaError_t launch_bucket_scan(const LaunchCtx& c, int64_t S, int32_t* cnt, int32_t* pos, WorkItem* work,
+                               int32_t* routed, int32_t* counters);
+cudaError_t launch_bucket_scatter(const LaunchCtx& c, unsigned long long* best, int64_t N,
+                                  const int32_t* scene_out, int32_t* pos, int32_t* item_tok);
 // K3
 struct ScoreArgs {
     int dtype;

@@ -47,9 +47,10 @@ __device__ __forceinline__ int segment_index(const GateSpec& gs, int64_t t) {
     return lo;
 }
 
-__device__ void gate_block(const GateSpec& gs, float* buf, int cap, int tpc) {
+// Gate CTA number `gi` (tokens [gi tpc, (gi + 1) tpc)).
+__device__ void gate_block(const GateSpec& gs, float* buf, int cap, int tpc, int64_t gi) {
     const int tid = threadIdx.x, warp = tid / 32, lane = tid % 32;
-    const int64_t tb = (int64_t)(blockIdx.x - 1) * tpc, te = min(gs.N, tb + tpc);
+    const int64_t tb = gi * tpc, te = min(gs.N, tb + tpc);
     if (tb >= te) return;  // uniform for the CTA
     const int64_t rb = gs.off[segment_index(gs, tb)], re = gs.off[segment_index(gs, te - 1) + 1];
     const bool staged = re - rb <= cap;  // uniform for the CTA
@@ -143,7 +144,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     pdl_trigger();
     pdl_wait();
     if (blockIdx.x > 0) {
-        gate_block(gate, reinterpret_cast<float*>(cnt), smem_bytes / 4, gate_tpc);
+        gate_block(gate, reinterpret_cast<float*>(cnt), smem_bytes / 4, gate_tpc, (int64_t)blockIdx.x - 1);
         return;
     }
     const int tid = threadIdx.x;
@@ -243,6 +244,155 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
+// ------------------------------------------------ large calls: three launches
+// The same work list and item-major token ids as k2_bucket, over all SMs.
+// Tokens of one scene in one warp are counted and placed with one atomic
+// (warp-aggregated), so a scene holding a sixth of the tokens (Zipf) costs a
+// few thousand atomics on its counter, not tens of thousands.
+
+// Per-scene counts.  CTAs [0, n_count) take token ranges of `per`; the CTAs
+// after them are gate CTAs (as in k2_bucket).
+__global__ void __launch_bounds__(kThreads, 1)
+    k2_count(unsigned long long* best, int64_t N, int S, int32_t* __restrict__ scene_out, int32_t* cnt, int64_t per,
+             int n_count, const __grid_constant__ GateSpec gate, int smem_bytes, int gate_tpc) {
+    extern __shared__ float stage[];
+    pdl_trigger();
+    pdl_wait();
+    if ((int)blockIdx.x >= n_count) {
+        gate_block(gate, stage, smem_bytes / 4, gate_tpc, (int64_t)blockIdx.x - n_count);
+        return;
+    }
+    const int lane = threadIdx.x % 32;
+    const int64_t t0 = (int64_t)blockIdx.x * per, t1 = min(N, t0 + per);
+    for (int64_t tb = t0; tb < t1; tb += kThreads) {
+        const int64_t t = tb + threadIdx.x;
+        const bool valid = t < t1;
+        const int32_t s = valid ? unpack_scene(best[t], S) : -1;
+        if (valid) scene_out[t] = s;
+        const uint32_t peers = __match_any_sync(0xFFFFFFFFu, s);
+        if (valid && lane == __ffs(peers) - 1) atomicAdd(&cnt[s], __popc(peers));
+    }
+}
+
+// The work list from the counts (one CTA), in rounds of 1,024 consecutive
+// scenes (thread i takes scene 1024 r + i, a block-wide scan per round and a
+// carry between rounds), so that every load and store of the round is
+// coalesced; pos[s] = the scene's first item_tok position; the counts are
+// zeroed for the next call.
+__global__ void __launch_bounds__(kThreads, 1)
+    k2_scan(int S, int32_t* cnt, int32_t* __restrict__ pos, WorkItem* __restrict__ work,
+            int32_t* __restrict__ routed, int32_t* __restrict__ counters) {
+    __shared__ int2 warp_buf[33];
+    __shared__ int max_bucket;
+    pdl_trigger();
+    pdl_wait();
+    const int tid = threadIdx.x;
+    if (tid == 0) max_bucket = 0;
+    int carry_items = 0, carry_routed = 0, mx = 0;
+    for (int r0 = 0; r0 < S; r0 += kThreads) {
+        const int s = r0 + tid;
+        const int c = s < S ? cnt[s] : 0;
+        if (s < S) cnt[s] = 0;
+        mx = max(mx, c);
+        int2 base, total;
+        block_exclusive_scan2(make_int2((c + kTokensPerItem - 1) / kTokensPerItem, c > 0), base, total, warp_buf);
+        const int wi = carry_items + base.x, slot = carry_routed + base.y;
+        if (s < S) {
+            pos[s] = wi * kTokensPerItem;
+            if (c > 0) {
+                routed[slot] = s;
+                for (int b = 0, i = wi; b < c; b += kTokensPerItem, ++i) {
+                    WorkItem w;
+                    w.scene = s;
+                    w.begin = i * kTokensPerItem;
+                    w.count = min(kTokensPerItem, c - b);
+                    w.slot = slot;
+                    work[i] = w;
+                }
+            }
+        }
+        carry_items += total.x;
+        carry_routed += total.y;
+        __syncthreads();  // warp_buf is reused by the next round
+    }
+    if (mx) atomicMax(&max_bucket, mx);
+    __syncthreads();
+    if (tid == 0) {
+        counters[0] = carry_items;
+        counters[1] = carry_routed;
+        counters[2] = max_bucket;
+        counters[3] = 0;  // level-2 work-taking counter
+    }
+}
+
+// The token ids into their items: a scene's k-th placed token lands in its
+// item k / 8, lane k % 8; the keys are cleared for the next call's argmax.
+__global__ void __launch_bounds__(kThreads)
+    k2_scatter(unsigned long long* best, int64_t N, const int32_t* scene_out, int32_t* pos,
+               int32_t* __restrict__ item_tok, int64_t per) {
+    pdl_trigger();
+    pdl_wait();
+    const int lane = threadIdx.x % 32;
+    const int64_t t0 = (int64_t)blockIdx.x * per, t1 = min(N, t0 + per);
+    for (int64_t tb = t0; tb < t1; tb += kThreads) {
+        const int64_t t = tb + threadIdx.x;
+        const bool valid = t < t1;
+        const int32_t s = valid ? scene_out[t] : -1;
+        const uint32_t peers = __match_any_sync(0xFFFFFFFFu, s);
+        const int leader = __ffs(peers) - 1;
+        int base = 0;
+        if (valid && lane == leader) base = atomicAdd(&pos[s], __popc(peers));
+        base = __shfl_sync(0xFFFFFFFFu, base, leader);
+        if (valid) {
+            item_tok[base + __popc(peers & ((1u << lane) - 1u))] = (int32_t)t;
+            best[t] = 0ull;
+        }
+    }
+}
+
+namespace {
+// Tokens per gate CTA: about two gate CTAs per SM, 8 to 32 tokens each.
+int gate_tokens_per_cta(const LaunchCtx& c, int64_t N) {
+    const int64_t want = (N + 2 * (int64_t)c.num_sms - 1) / (2 * (int64_t)c.num_sms);
+    return (int)std::min<int64_t>(kGateMaxTokens, std::max<int64_t>(8, want));
+}
+// Token ranges of the count and scatter launches: one range per SM at most.
+int64_t big_ranges(const LaunchCtx& c, int64_t N) {
+    return std::max<int64_t>(1, std::min<int64_t>(c.num_sms, (N + kThreads - 1) / kThreads));
+}
+}  // namespace
+
+cudaError_t launch_bucket_count(const LaunchCtx& c, unsigned long long* best, int64_t N, int64_t S,
+                                int32_t* scene_out, int32_t* cnt, const GateSpec* gate) {
+    GateSpec gs;
+    if (gate) {
+        gs = *gate;
+    } else {
+        memset(&gs, 0, sizeof(gs));
+    }
+    const int64_t nr = big_ranges(c, N);
+    const int64_t per = (N + nr - 1) / nr;
+    const int n_count = (int)((N + per - 1) / per);
+    const int tpc = gate_tokens_per_cta(c, N);
+    const int gate_ctas = gate ? (int)((N + tpc - 1) / tpc) : 0;
+    const int smem = gate ? kGateStage : 0;
+    return launch_pdl(k2_count, dim3(n_count + gate_ctas), dim3(kThreads), (size_t)smem, c.stream, best, N, (int)S,
+                      scene_out, cnt, per, n_count, gs, smem, tpc);
+}
+
+cudaError_t launch_bucket_scan(const LaunchCtx& c, int64_t S, int32_t* cnt, int32_t* pos, WorkItem* work,
+                               int32_t* routed, int32_t* counters) {
+    return launch_pdl(k2_scan, dim3(1), dim3(kThreads), 0, c.stream, (int)S, cnt, pos, work, routed, counters);
+}
+
+cudaError_t launch_bucket_scatter(const LaunchCtx& c, unsigned long long* best, int64_t N,
+                                  const int32_t* scene_out, int32_t* pos, int32_t* item_tok) {
+    const int64_t nr = big_ranges(c, N);
+    const int64_t per = (N + nr - 1) / nr;
+    const int grid = (int)((N + per - 1) / per);
+    return launch_pdl(k2_scatter, dim3(grid), dim3(kThreads), 0, c.stream, best, N, scene_out, pos, item_tok, per);
+}
+
 cudaError_t launch_bucket(const LaunchCtx& c, unsigned long long* best, int64_t N, int64_t S,
                           int32_t* scene_out, int32_t* item_tok, WorkItem* work, int32_t* routed, int32_t* counters,
                           const GateSpec* gate) {
@@ -252,9 +402,7 @@ cudaError_t launch_bucket(const LaunchCtx& c, unsigned long long* best, int64_t 
     } else {
         memset(&gs, 0, sizeof(gs));
     }
-    // Tokens per gate CTA: about two gate CTAs per SM, 8 to 32 tokens each.
-    const int64_t want = (N + 2 * (int64_t)c.num_sms - 1) / (2 * (int64_t)c.num_sms);
-    const int tpc = (int)std::min<int64_t>(kGateMaxTokens, std::max<int64_t>(8, want));
+    const int tpc = gate_tokens_per_cta(c, N);
     const int gate_ctas = gate ? (int)((N + tpc - 1) / tpc) : 0;
     const int smem = (int)std::max<int64_t>(S * (int64_t)sizeof(int), gate ? kGateStage : 0);
     return launch_pdl(k2_bucket, dim3(1 + gate_ctas), dim3(kThreads), (size_t)smem, c.stream, best, N, (int)S,

@@ -41,7 +41,7 @@ lookme_status fail(lookme_status st, const char* fmt, ...) {
 const char* kKernelNames[KID_COUNT] = {"prep",         "route_tc", "route_simt",    "bucket",
                                        "score",        "select",   "inject",        "stage",
                                        "centroid_mean", "inv_cnorm", "route_decode", "select_inject",
-                                       "tile_keys"};
+                                       "tile_keys",    "bucket_count", "bucket_scan", "bucket_scatter"};
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point, so the
 // library does not link libcuda directly.
@@ -135,6 +135,8 @@ struct lookme_table {
     int32_t* rec_t = nullptr;    // injection records by kept slot: token id,
     int32_t* rec_row = nullptr;  // value rows and weights (kRecMaxTopK per slot)
     float* rec_w = nullptr;
+    int32_t* scene_cnt = nullptr;  // large calls' bucketing: per-scene counts (zero between calls)
+    int32_t* scene_pos = nullptr;  // and running item_tok positions
     uint32_t* status = nullptr;   // persistent device status word
     int64_t last_tokens = -1;
     int64_t last_staged_bytes = 0;
@@ -228,6 +230,8 @@ lookme_status ensure_scratch(lookme_table* t, int64_t n, cudaStream_t s) {
     const size_t o_rec_t = take(cap * sizeof(int32_t));
     const size_t o_rec_row = take(cap * kRecMaxTopK * sizeof(int32_t));
     const size_t o_rec_w = take(cap * kRecMaxTopK * sizeof(float));
+    const size_t o_scnt = take(S * sizeof(int32_t));
+    const size_t o_spos = take(S * sizeof(int32_t));
     void* buf = nullptr;
     if (cudaDeviceSynchronize() != cudaSuccess || cudaMalloc(&buf, off) != cudaSuccess) {
         cudaGetLastError();
@@ -249,6 +253,8 @@ lookme_status ensure_scratch(lookme_table* t, int64_t n, cudaStream_t s) {
     t->rec_t = reinterpret_cast<int32_t*>(b + o_rec_t);
     t->rec_row = reinterpret_cast<int32_t*>(b + o_rec_row);
     t->rec_w = reinterpret_cast<float*>(b + o_rec_w);
+    t->scene_cnt = reinterpret_cast<int32_t*>(b + o_scnt);
+    t->scene_pos = reinterpret_cast<int32_t*>(b + o_spos);
     t->last_tokens = -1;
     if (cudaMemset(buf, 0, off) != cudaSuccess) return cuda_fail(t, cudaGetLastError(), "scratch memset");
     return LOOKME_OK;
@@ -549,10 +555,28 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
         });
     }
     if (st != LOOKME_OK) return st;
-    st = launch(t, s, KID_BUCKET, [&] {
-        return launch_bucket(ctx, t->best, N, d.n_scenes, scene_out, t->item_tok, t->work, t->routed, t->counters,
-                             gate);
-    });
+    // Large calls without the gate: the bucketing over all SMs in three
+    // launches.  With the gate, its CTAs dominate and run beside the
+    // single-CTA sort, which is then the faster choice.
+    if (N <= kBucketOneCtaTokens || gate) {
+        st = launch(t, s, KID_BUCKET, [&] {
+            return launch_bucket(ctx, t->best, N, d.n_scenes, scene_out, t->item_tok, t->work, t->routed,
+                                 t->counters, gate);
+        });
+    } else {
+        st = launch(t, s, KID_BUCKET_COUNT, [&] {
+            return launch_bucket_count(ctx, t->best, N, d.n_scenes, scene_out, t->scene_cnt, gate);
+        });
+        if (st == LOOKME_OK)
+            st = launch(t, s, KID_BUCKET_SCAN, [&] {
+                return launch_bucket_scan(ctx, d.n_scenes, t->scene_cnt, t->scene_pos, t->work, t->routed,
+                                          t->counters);
+            });
+        if (st == LOOKME_OK)
+            st = launch(t, s, KID_BUCKET_SCATTER, [&] {
+                return launch_bucket_scatter(ctx, t->best, N, scene_out, t->scene_pos, t->item_tok);
+            });
+    }
     if (st != LOOKME_OK) return st;
     const bool staged = d.residency == LOOKME_RES_HOST_STAGED;
     if (staged) {

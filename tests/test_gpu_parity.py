@@ -293,6 +293,21 @@ def test_lookup_inject_many_items(oracle, lookme_lib, extra):
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+@pytest.mark.parametrize("fused", [False, True])
+def test_large_call_bucketing(oracle, lookme_lib, dtype, fused):
+    """More than 8,192 tokens (the bucketing runs as three launches over all
+    SMs) in 64 scenes of ~140 tokens each, so every scene splits into many
+    work items, with three segments for the gate."""
+    w = W.small(f"bigcall_{dtype}", dtype=dtype, n_tokens=9000, n_scenes=64, n_prims=32, d_key=64, d_value=64,
+                top_k=4, keep_ratio=0.25, n_segments=3)
+    rep = {}
+    run_case(oracle, lookme_lib, w, fused=fused, report=rep)
+    counts = np.bincount(rep["scene"], minlength=w.n_scenes)
+    assert rep["stats"]["n_work_items"] == int(((counts + 7) // 8).sum())
+    assert rep["stats"]["n_routed_scenes"] == int((counts > 0).sum())
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
 @pytest.mark.parametrize("name", ["s2", "s3", "s6", "s8", "layers"])
 def test_lookup_inject_matches_separate_calls(lookme_lib, dtype, name):
     """lookme_lookup_inject gives bit-identical results to lookme_lookup +
