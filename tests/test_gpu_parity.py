@@ -307,6 +307,18 @@ def test_large_call_bucketing(oracle, lookme_lib, dtype, fused):
     assert rep["stats"]["n_routed_scenes"] == int((counts > 0).sum())
 
 
+def test_large_call_bucketing_host_staged(oracle, lookme_lib):
+    """The three-launch bucketing feeding the staging of a pinned-host table
+    (the routed-scene list and counts come from its scan)."""
+    w = W.small("bigcall_host", n_tokens=9000, n_scenes=96, n_prims=32, d_key=64, d_value=64, top_k=4,
+                keep_ratio=0.25, residency="host")
+    rep = {}
+    run_case(oracle, lookme_lib, w, report=rep)
+    counts = np.bincount(rep["scene"], minlength=w.n_scenes)
+    assert rep["stats"]["n_routed_scenes"] == int((counts > 0).sum())
+    assert rep["stats"]["staged_bytes"] == int((counts > 0).sum()) * w.n_prims * w.d_key * 2
+
+
 @pytest.mark.parametrize("dtype", ["bf16", "fp32"])
 @pytest.mark.parametrize("name", ["s2", "s3", "s6", "s8", "layers"])
 def test_lookup_inject_matches_separate_calls(lookme_lib, dtype, name):
