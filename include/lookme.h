@@ -167,7 +167,9 @@ lookme_status lookme_inject(lookme_table* table, const int32_t* scene, const int
  * these queries; mask_out (device [n_tokens] uint8, or NULL) receives the
  * gate.  With at most 64 segments of at most 8,192 tokens, the gate is
  * decided during the lookup (beside the bucketing) and the injection visits
- * only the kept tokens.  Errors: those of lookme_lookup and lookme_inject
+ * only the kept tokens; on HBM-resident bf16 tables with top_k <= 16 the
+ * level-2 kernel hands each kept token's value rows and weights to the
+ * injection directly.  Errors: those of lookme_lookup and lookme_inject
  * (the injection arguments are checked before anything runs). */
 lookme_status lookme_lookup_inject(lookme_table* table, const void* queries, int64_t n_tokens, int32_t top_k,
                                    const float* priority, const int64_t* seg_offsets, int32_t n_seg,
