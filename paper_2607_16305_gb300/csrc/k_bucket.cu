@@ -154,6 +154,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Both sweeps over the tokens issue kB keys per thread before using any
     // (one round trip per batch, not per token); the scenes of a thread's
     // first batch stay in registers for the second sweep.
+    // A batch stops at its last valid token, so a call of at most 1,024
+    // tokens runs one slot per thread, not eight mostly idle ones.
     constexpr int kB = 8;
     int32_t sc[kB];
     for (int64_t t0 = tid; t0 < N; t0 += (int64_t)kB * kThreads) {
@@ -161,17 +163,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int u = 0; u < kB; ++u) {
             const int64_t t = t0 + (int64_t)u * kThreads;
-            key[u] = t < N ? best[t] : 0ull;
+            if (t >= N) break;
+            key[u] = best[t];
         }
 #pragma unroll
         for (int u = 0; u < kB; ++u) {
             const int64_t t = t0 + (int64_t)u * kThreads;
+            if (t >= N) break;
             const int32_t s = unpack_scene(key[u], S);
             if (t0 == tid) sc[u] = s;
-            if (t < N) {
-                scene_out[t] = s;
-                atomicAdd(&cnt[s], 1);
-            }
+            scene_out[t] = s;
+            atomicAdd(&cnt[s], 1);
         }
     }
     __syncthreads();
@@ -227,19 +229,22 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int u = 0; u < kB; ++u) {
                 const int64_t t = t0 + (int64_t)u * kThreads;
-                key[u] = t < N ? best[t] : 0ull;
+                if (t >= N) break;
+                key[u] = best[t];
             }
 #pragma unroll
-            for (int u = 0; u < kB; ++u) s[u] = unpack_scene(key[u], S);
+            for (int u = 0; u < kB; ++u) {
+                if (t0 + (int64_t)u * kThreads >= N) break;
+                s[u] = unpack_scene(key[u], S);
+            }
         }
 #pragma unroll
         for (int u = 0; u < kB; ++u) {
             const int64_t t = t0 + (int64_t)u * kThreads;
-            if (t < N) {
-                best[t] = 0ull;
-                const int pos = atomicAdd(&cnt[s[u]], 1);
-                item_tok[pos] = (int32_t)t;
-            }
+            if (t >= N) break;
+            best[t] = 0ull;
+            const int pos = atomicAdd(&cnt[s[u]], 1);
+            item_tok[pos] = (int32_t)t;
         }
     }
 }
