@@ -148,23 +148,32 @@ __global__ void __launch_bounds__(kThreads, 1)
         return;
     }
     const int tid = threadIdx.x;
-    for (int s = tid; s < S; s += kThreads) cnt[s] = 0;
-    if (tid == 0) max_bucket = 0;
-    __syncthreads();
     // Both sweeps over the tokens issue kB keys per thread before using any
     // (one round trip per batch, not per token); the scenes of a thread's
     // first batch stay in registers for the second sweep.
     // A batch stops at its last valid token, so a call of at most 1,024
     // tokens runs one slot per thread, not eight mostly idle ones.
     constexpr int kB = 8;
+    unsigned long long key[kB];
+    // The first batch is requested before the counters are cleared.
+#pragma unroll
+    for (int u = 0; u < kB; ++u) {
+        const int64_t t = tid + (int64_t)u * kThreads;
+        if (t >= N) break;
+        key[u] = best[t];
+    }
+    for (int s = tid; s < S; s += kThreads) cnt[s] = 0;
+    if (tid == 0) max_bucket = 0;
+    __syncthreads();
     int32_t sc[kB];
     for (int64_t t0 = tid; t0 < N; t0 += (int64_t)kB * kThreads) {
-        unsigned long long key[kB];
+        if (t0 != tid) {
 #pragma unroll
-        for (int u = 0; u < kB; ++u) {
-            const int64_t t = t0 + (int64_t)u * kThreads;
-            if (t >= N) break;
-            key[u] = best[t];
+            for (int u = 0; u < kB; ++u) {
+                const int64_t t = t0 + (int64_t)u * kThreads;
+                if (t >= N) break;
+                key[u] = best[t];
+            }
         }
 #pragma unroll
         for (int u = 0; u < kB; ++u) {
@@ -191,7 +200,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     int2 base, total;
     block_exclusive_scan2(mine, base, total, warp_buf);
-    if (mx) atomicMax(&max_bucket, mx);
+    // One shared atomic per warp, not one per routed scene on a single word.
+    mx = __reduce_max_sync(0xFFFFFFFFu, mx);
+    if (tid % 32 == 0 && mx) atomicMax(&max_bucket, mx);
 
     int wi = base.x, slot = base.y;
     for (int s = s0; s < s1; ++s) {
@@ -320,7 +331,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         carry_routed += total.y;
         __syncthreads();  // warp_buf is reused by the next round
     }
-    if (mx) atomicMax(&max_bucket, mx);
+    mx = __reduce_max_sync(0xFFFFFFFFu, mx);
+    if (tid % 32 == 0 && mx) atomicMax(&max_bucket, mx);
     __syncthreads();
     if (tid == 0) {
         counters[0] = carry_items;
