@@ -32,7 +32,7 @@ def launches(csv_path, out, cmd):
             us = v / 1000.0 if unit in ("nsecond", "ns") else v * 1000.0 if unit in ("msecond", "ms") else v
             per[x["Kernel Name"].split("(")[0].replace("void ", "")].append(us)
     total = sum(sum(v) for k, v in per.items() if "lookme" in k)
-    lines = [f"# ncu launch list: {out.split('/')[-1]}", "", "Command (run under gpurun on one GB300):", "",
+    lines = [f"# ncu launch list: {out.split('/')[-1]}", "", "Command (run on one GB300):", "",
              f"    {cmd}", "",
              "Per-launch times are cold-cache and serialised (ncu); compare shares, not absolutes.", "",
              "| kernel | launches | total us | mean us | share of library time |", "|---|---|---|---|---|"]
@@ -68,7 +68,7 @@ def kernel(rep, out, cmd, src, alg_bytes):
     stalls = sorted(((float(get[h][0].replace(",", "")), h) for h in get
                      if h.startswith("smsp__pcsamp_warps_issue_stalled") and not h.endswith("not_issued")
                      and get[h][0].replace(",", "").replace(".", "").isdigit()), reverse=True)[:6]
-    lines = [f"# ncu --set full: {name}", "", "Command (run under gpurun on one GB300):", "", f"    {cmd}", "",
+    lines = [f"# ncu --set full: {name}", "", "Command (run on one GB300):", "", f"    {cmd}", "",
              f"source_sha: {sha}", f"traffic_bytes_per_launch: {rd + wr:.0f}", "",
              "| quantity | value |", "|---|---|",
              f"| duration (ncu, cold L2, clocks uncontrolled) | {dur * 1e6:.2f} us |",
