@@ -73,22 +73,30 @@ def load_peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
 
 
-def kernel_source_sha():
+# The sources each profiled kernel is built from (the hash ties an ncu summary to them).
+KERNEL_SOURCES = {
+    "score": ["k_score_tc.cu", "score_tc.cuh", "topk.cuh", "sm100.cuh"],
+    "step": ["k_step.cu", "score_tc.cuh", "topk.cuh", "sm100.cuh"],
+}
+
+
+def kernel_source_sha(kernel="step"):
     h = hashlib.sha256()
-    with open(os.path.join(ROOT, "paper_2607_16305_gb300", "csrc", "k_score_tc.cu"), "rb") as f:
-        h.update(f.read())
+    for f in KERNEL_SOURCES[kernel]:
+        with open(os.path.join(ROOT, "paper_2607_16305_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload):
-    """DRAM bytes per launch of the scoring kernel from the committed ncu summary, if it is current."""
-    p = os.path.join(ROOT, "profiles", f"ncu_score_{workload}.md")
+def profiled_traffic(kernel, workload):
+    """DRAM bytes per launch of `kernel` from its committed ncu summary, if that summary is current."""
+    p = os.path.join(ROOT, "profiles", f"ncu_{kernel}_{workload}.md")
     if not os.path.exists(p):
         return None
     txt = open(p).read()
     m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt)
     s = re.search(r"source_sha:\s*([0-9a-f]+)", txt)
-    if not m or not s or s.group(1) != kernel_source_sha():
+    if not m or not s or s.group(1) != kernel_source_sha(kernel):
         return None
     return float(m.group(1))
 
@@ -336,7 +344,7 @@ def run_lookme(args, w, ws, rank, local):
                      "achieved": achieved, "peak": hbm, "unit": "GB/s",
                      "frac": achieved / hbm if achieved else None, "peak_source": peak_kind,
                      "algorithmic_bytes": ab["score"], "mean_ms": score_ms,
-                     "traffic": profiled_traffic(w.name)},
+                     "traffic": profiled_traffic("score", w.name)},
         "step_roofline": {"bound": "hbm", "algorithmic_bytes": ab["step"], "achieved": step_gbs, "peak": hbm,
                           "unit": "GB/s", "frac": step_gbs / hbm, "roofline_us": ab["step"] / hbm / 1e3},
         "eager_ms_per_step": eager_ms,

@@ -30,6 +30,7 @@ enum KernelId : int32_t {
     KID_BUCKET_COUNT = 13,    // K2 for large calls: per-scene counts (+ gate CTAs)
     KID_BUCKET_SCAN = 14,     // K2 for large calls: work list from the counts
     KID_BUCKET_SCATTER = 15,  // K2 for large calls: token ids into their items
+    KID_STEP = 16,            // K1 + K2 + K3 (+ gate and K4): the fused step on tcgen05
     KID_COUNT
 };
 
@@ -37,6 +38,7 @@ enum KernelId : int32_t {
 constexpr uint32_t STATUS_WAIT_TIMEOUT = 1u;
 constexpr uint32_t STATUS_IN_ROUTE = 2u;  // set with STATUS_WAIT_TIMEOUT by the level-1 kernel
 constexpr uint32_t STATUS_IN_SCORE = 4u;  // set with STATUS_WAIT_TIMEOUT by a level-2 kernel
+constexpr uint32_t STATUS_IN_STEP = 8u;   // set with STATUS_WAIT_TIMEOUT by the fused step kernel
 
 // ------------------------------------------------------------ element access
 __device__ __forceinline__ float to_f32(float x) { return x; }
@@ -265,12 +267,67 @@ cudaError_t launch_select_inject(const LaunchCtx& c, const InjectArgs& a, const 
 cudaError_t launch_stage(const LaunchCtx& c, const void* keys_host_mapped, void* slots, int64_t block_bytes,
                          int64_t n_slots, const int32_t* routed, const int32_t* counters);
 
+// ------------------------------------------------------------- fused step
+// Routing, bucketing, level 2, the injection gate and the injection in one
+// launch of one CTA per SM (bf16 tables in HBM, N <= kStepMaxTokens,
+// top_k <= kRecMaxTopK).  The call-to-call state it keeps in device memory
+// (zero when first allocated): the epoch whose parity picks the argmax-key
+// buffer and the grid-barrier counter of a call, and the exit ticket.
+constexpr int64_t kStepMaxTokens = 8192;
+struct StepState {
+    uint32_t epoch;
+    uint32_t exit_cnt;
+    uint32_t bar[2];
+    uint32_t pad[60];
+    unsigned long long best[2][kStepMaxTokens];
+};
+struct StepArgs {
+    int64_t N, S, P;
+    int dk, dv, top_k;
+    float scale;
+    const void* q;           // [N][d_k] bf16
+    const void* keys_tiled;  // the level-2 tile layout, one block per scene
+    int64_t block_bytes;
+    const void* values;      // [S][P][d_v] bf16
+    const float* inv_cnorm;
+    const float* bias;       // or null
+    int32_t* scene_out;
+    int32_t* prim_out;
+    float* weight_out;
+    float* qnorm;            // [N] scratch: the query norms (default gate priority)
+    float* qnorm_out;        // or null
+    // gate and injection; gate = 0 is a lookup without injection
+    int gate;
+    int n_seg;
+    const float* priority;   // or null: the query norms
+    uint8_t* mask_out;       // or null
+    int64_t seg_off[kMaxGateSegments + 1];
+    int64_t seg_r[kMaxGateSegments];
+    int n_layers;
+    void* hidden[LOOKME_MAX_LAYERS];
+    // scratch
+    StepState* state;
+    WorkItem* work;          // >= N + S entries
+    int32_t* item_tok;       // kTokensPerItem per work entry
+    int32_t* counters;       // [0] work items, [1] routed scenes, [2] largest bucket
+    uint32_t* status;
+    // kept tokens past a CTA's on-chip queue: their value rows and weights by
+    // token id ([N][kRecMaxTopK]) and their ids (kTokensPerItem per work entry)
+    int32_t* rec_row;
+    float* rec_w;
+    int32_t* ovf_tok;
+};
+// Whether the fused step handles this table shape (shared memory, TMEM).
+bool step_shape_supported(int64_t N, int64_t S, int64_t P, int dk, int dv, int num_sms);
+cudaError_t launch_step(const LaunchCtx& c, const void* tmap_q, const void* const tmap_c[3], const StepArgs& a);
+
 // Raise the dynamic shared-memory limits of the kernels that need more than
 // 48 KB (per device; call with the device current).
 cudaError_t configure_route_kernels();
 cudaError_t configure_bucket_kernel();
 cudaError_t configure_score_kernels();
 cudaError_t configure_score_tc_kernel();
+cudaError_t configure_step_kernel();
 // load-time
 cudaError_t launch_centroid_mean(const LaunchCtx& c, int dtype, const void* keys, int64_t n, int64_t P, int dk,
                                  void* cent);

@@ -41,7 +41,8 @@ lookme_status fail(lookme_status st, const char* fmt, ...) {
 const char* kKernelNames[KID_COUNT] = {"prep",         "route_tc", "route_simt",    "bucket",
                                        "score",        "select",   "inject",        "stage",
                                        "centroid_mean", "inv_cnorm", "route_decode", "select_inject",
-                                       "tile_keys",    "bucket_count", "bucket_scan", "bucket_scatter"};
+                                       "tile_keys",    "bucket_count", "bucket_scan", "bucket_scatter",
+                                       "step"};
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point, so the
 // library does not link libcuda directly.
@@ -103,6 +104,7 @@ struct lookme_table {
     int num_sms = 0;
     bool tc_route = false;  // level 1 on tcgen05
     bool tc_score = false;  // level 2 on tcgen05
+    bool use_step = false;  // whole calls as one fused launch where the shape allows
     int64_t kblock = 0;     // bytes of one scene's stored key block (tiled when tc_score)
 
     // storage
@@ -137,6 +139,8 @@ struct lookme_table {
     float* rec_w = nullptr;
     int32_t* scene_cnt = nullptr;  // large calls' bucketing: per-scene counts (zero between calls)
     int32_t* scene_pos = nullptr;  // and running item_tok positions
+    StepState* step = nullptr;     // the fused step's call-to-call state (zero at allocation)
+    int32_t* step_ovf = nullptr;   // the fused step's kept tokens past a CTA's on-chip queue
     uint32_t* status = nullptr;   // persistent device status word
     int64_t last_tokens = -1;
     int64_t last_staged_bytes = 0;
@@ -232,6 +236,8 @@ lookme_status ensure_scratch(lookme_table* t, int64_t n, cudaStream_t s) {
     const size_t o_rec_w = take(cap * kRecMaxTopK * sizeof(float));
     const size_t o_scnt = take(S * sizeof(int32_t));
     const size_t o_spos = take(S * sizeof(int32_t));
+    const size_t o_step = take(sizeof(StepState));
+    const size_t o_sovf = take((cap + S) * kTokensPerItem * sizeof(int32_t));
     void* buf = nullptr;
     if (cudaDeviceSynchronize() != cudaSuccess || cudaMalloc(&buf, off) != cudaSuccess) {
         cudaGetLastError();
@@ -255,6 +261,8 @@ lookme_status ensure_scratch(lookme_table* t, int64_t n, cudaStream_t s) {
     t->rec_w = reinterpret_cast<float*>(b + o_rec_w);
     t->scene_cnt = reinterpret_cast<int32_t*>(b + o_scnt);
     t->scene_pos = reinterpret_cast<int32_t*>(b + o_spos);
+    t->step = reinterpret_cast<StepState*>(b + o_step);
+    t->step_ovf = reinterpret_cast<int32_t*>(b + o_sovf);
     t->last_tokens = -1;
     if (cudaMemset(buf, 0, off) != cudaSuccess) return cuda_fail(t, cudaGetLastError(), "scratch memset");
     return LOOKME_OK;
@@ -355,11 +363,19 @@ lookme_status lookme_table_create(const lookme_table_desc* desc, lookme_table** 
     if (const char* env = getenv("LOOKME_SCORE")) {
         if (strcmp(env, "simt") == 0) t->tc_score = false;
     }
+    // LOOKME_STEP=on runs whole calls as one launch of the fused step kernel
+    // where the shape allows (it is correct, but measured slower than the
+    // separate kernels on this GB300, so it is not the default).
+    t->use_step = false;
+    if (const char* env = getenv("LOOKME_STEP")) {
+        if (strcmp(env, "on") == 0) t->use_step = t->tc_route && t->tc_score;
+    }
     t->loaded.assign(d.n_scenes, 0);
 
     cudaError_t e;
     if ((e = configure_route_kernels()) != cudaSuccess || (e = configure_bucket_kernel()) != cudaSuccess ||
-        (e = configure_score_kernels()) != cudaSuccess || (e = configure_score_tc_kernel()) != cudaSuccess) {
+        (e = configure_score_kernels()) != cudaSuccess || (e = configure_score_tc_kernel()) != cudaSuccess ||
+        (e = configure_step_kernel()) != cudaSuccess) {
         destroy_table(t);
         return fail(LOOKME_ERR_CUDA, "kernel configuration: %s", cudaGetErrorString(e));
     }
@@ -507,12 +523,9 @@ lookme_status lookme_load_scenes(lookme_table* t, int64_t scene_begin, int64_t n
 
 namespace {
 
-// lookme_lookup; with gate the bucketing kernel also computes the injection gate.
-lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32_t top_k, int32_t* scene_out,
-                          int32_t* prim_out, float* weight_out, float* qnorm_out, lookme_stream stream,
-                          const GateSpec* gate, const void* hidden0 = nullptr, bool records = false) {
-    lookme_status st = check_table(t);
-    if (st != LOOKME_OK) return st;
+// Argument checks shared by every lookup entry point.
+lookme_status check_lookup(const lookme_table* t, const void* queries, int64_t N, int32_t top_k,
+                           const int32_t* scene_out, const int32_t* prim_out, const float* weight_out) {
     const lookme_table_desc& d = t->d;
     if (N < 0 || N > INT32_MAX / 2) return fail(LOOKME_ERR_INVALID_ARG, "n_tokens %lld out of range", (long long)N);
     if (top_k < 1 || top_k > LOOKME_MAX_TOP_K || top_k > d.n_prims)
@@ -525,9 +538,93 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
     if (d.residency == LOOKME_RES_HOST_STAGED && std::min<int64_t>(N, d.n_scenes) > t->n_slots)
         return fail(LOOKME_ERR_UNSUPPORTED, "up to %lld routed scenes but only %lld staging slots",
                     (long long)std::min<int64_t>(N, d.n_scenes), (long long)t->n_slots);
+    return LOOKME_OK;
+}
+
+// Whether a call of N tokens (with n_seg gate segments) runs as the fused step.
+bool step_eligible(const lookme_table* t, int64_t N, int32_t top_k, int n_seg) {
+    const lookme_table_desc& d = t->d;
+    return t->use_step && d.residency == LOOKME_RES_DEVICE && N >= 1 && N <= kStepMaxTokens &&
+           top_k <= kRecMaxTopK && n_seg <= kMaxGateSegments &&
+           step_shape_supported(N, d.n_scenes, d.n_prims, (int)d.d_key, (int)d.d_value, t->num_sms);
+}
+
+// The whole call as one launch of the fused step kernel.  With gate_off
+// (the gate's segment offsets, n_seg + 1 of them) the call also decides the
+// gate and injects; without it, it is a lookup.  Arguments are checked.
+lookme_status run_step(lookme_table* t, cudaStream_t s, const void* queries, int64_t N, int32_t top_k,
+                       int32_t* scene_out, int32_t* prim_out, float* weight_out, float* qnorm_out,
+                       const int64_t* gate_off, int n_seg, double keep_ratio, const float* priority,
+                       void* const* hidden, int32_t n_layers, uint8_t* mask_out) {
+    const lookme_table_desc& d = t->d;
+    lookme_status st;
+    if ((st = ensure_scratch(t, N, s)) != LOOKME_OK) return st;
+    CUtensorMap mq;
+    if (!encode_bf16_2d(&mq, queries, N, d.d_key, 128))
+        return fail(LOOKME_ERR_CUDA, "cuTensorMapEncodeTiled failed for the queries");
+    const void* mc[3] = {&t->tmap_c[0], &t->tmap_c[1], &t->tmap_c[2]};
+    StepArgs a;
+    memset(&a, 0, sizeof(a));
+    a.N = N;
+    a.S = d.n_scenes;
+    a.P = d.n_prims;
+    a.dk = (int)d.d_key;
+    a.dv = (int)d.d_value;
+    a.top_k = top_k;
+    a.scale = (float)(1.0 / std::sqrt((double)d.d_key));
+    a.q = queries;
+    a.keys_tiled = t->keys;
+    a.block_bytes = t->kblock;
+    a.values = t->values;
+    a.inv_cnorm = t->inv_cnorm;
+    a.bias = t->has_bias ? t->bias : nullptr;
+    a.scene_out = scene_out;
+    a.prim_out = prim_out;
+    a.weight_out = weight_out;
+    a.qnorm = t->qnorm;
+    a.qnorm_out = qnorm_out;
+    a.gate = gate_off ? 1 : 0;
+    a.n_seg = gate_off ? n_seg : 1;
+    a.priority = priority;
+    a.mask_out = mask_out;
+    if (gate_off) {
+        for (int i = 0; i <= n_seg; ++i) a.seg_off[i] = gate_off[i];
+        for (int i = 0; i < n_seg; ++i)
+            a.seg_r[i] = (int64_t)std::floor((double)(gate_off[i + 1] - gate_off[i]) * keep_ratio);
+        a.n_layers = n_layers;
+        for (int l = 0; l < n_layers; ++l) a.hidden[l] = hidden[l];
+    } else {
+        a.seg_off[1] = N;
+    }
+    a.state = t->step;
+    a.work = t->work;
+    a.item_tok = t->item_tok;
+    a.counters = t->counters;
+    a.status = t->status;
+    a.rec_row = t->rec_row;
+    a.rec_w = t->rec_w;
+    a.ovf_tok = t->step_ovf;
+    LaunchCtx ctx{s, t->num_sms};
+    st = launch(t, s, KID_STEP, [&] { return launch_step(ctx, &mq, mc, a); });
+    if (st != LOOKME_OK) return st;
+    t->last_tokens = N;
+    return LOOKME_OK;
+}
+
+// lookme_lookup; with gate the bucketing kernel also computes the injection gate.
+lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32_t top_k, int32_t* scene_out,
+                          int32_t* prim_out, float* weight_out, float* qnorm_out, lookme_stream stream,
+                          const GateSpec* gate, const void* hidden0 = nullptr, bool records = false) {
+    lookme_status st = check_table(t);
+    if (st != LOOKME_OK) return st;
+    const lookme_table_desc& d = t->d;
+    if ((st = check_lookup(t, queries, N, top_k, scene_out, prim_out, weight_out)) != LOOKME_OK) return st;
     if (N == 0) return LOOKME_OK;
     DeviceGuard guard(d.device);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (!gate && step_eligible(t, N, top_k, 1))
+        return run_step(t, s, queries, N, top_k, scene_out, prim_out, weight_out, qnorm_out, nullptr, 1, 0.0, nullptr,
+                        nullptr, 0, nullptr);
     if ((st = ensure_scratch(t, N, s)) != LOOKME_OK) return st;
     LaunchCtx ctx{s, t->num_sms};
     const int dk = (int)d.d_key;
@@ -734,6 +831,13 @@ lookme_status lookme_lookup_inject(lookme_table* t, const void* queries, int64_t
     if (st != LOOKME_OK) return st;
     InjectPlan plan;
     if ((st = plan_inject(t, N, top_k, seg_offsets, n_seg, keep_ratio, hidden, n_layers, plan)) != LOOKME_OK) return st;
+    if (step_eligible(t, N, top_k, plan.n_seg)) {
+        // Everything in one launch of the fused step kernel.
+        if ((st = check_lookup(t, queries, N, top_k, scene_out, prim_out, weight_out)) != LOOKME_OK) return st;
+        DeviceGuard guard(t->d.device);
+        return run_step(t, static_cast<cudaStream_t>(stream), queries, N, top_k, scene_out, prim_out, weight_out,
+                        nullptr, plan.off.data(), plan.n_seg, keep_ratio, priority, hidden, n_layers, mask_out);
+    }
     const bool gate_in_lookup = N > 0 && plan.n_seg <= kMaxGateSegments && plan.max_seg <= kFusedMaxSegment;
     if (!gate_in_lookup) {
         // The two calls in sequence; with PDL the injection kernel's launch

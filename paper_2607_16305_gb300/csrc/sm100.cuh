@@ -44,31 +44,36 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     return ok != 0;
 }
 
+// The spinning part of mbar_wait, out of line: one copy of its code serves
+// every wait (the kernels keep their code small enough to stay in the
+// instruction cache from one launch to the next).
+static __device__ __noinline__ bool mbar_spin(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                              uint64_t timeout_ns) {
+    const uint64_t t0 = globaltimer_ns();
+    for (;;) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (abort && *abort) return false;
+        if (globaltimer_ns() - t0 > timeout_ns) {
+            if (abort) *abort = 1;
+            return false;
+        }
+    }
+}
+
 // Wait for the phase with the given parity to complete.  Gives up after
 // timeout_ns or as soon as *abort is set; on a timeout it sets *abort.
 // Returns true when the phase completed.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
                                           uint64_t timeout_ns) {
     if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = globaltimer_ns();
-    for (;;) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if (*abort) return false;
-        if (globaltimer_ns() - t0 > timeout_ns) {
-            *abort = 1;
-            return false;
-        }
-    }
+    return mbar_spin(bar, parity, abort, timeout_ns);
 }
 
 // Bounded wait that ignores the abort flag: used while draining in-flight
 // copies and MMAs before a CTA exits.
 __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity, uint64_t timeout_ns) {
-    const uint64_t t0 = globaltimer_ns();
-    while (!mbar_try_wait(bar, parity)) {
-        if (globaltimer_ns() - t0 > timeout_ns) return false;
-    }
-    return true;
+    if (mbar_try_wait(bar, parity)) return true;
+    return mbar_spin(bar, parity, nullptr, timeout_ns);
 }
 
 // ------------------------------------------------------------ bulk copies
