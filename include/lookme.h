@@ -229,7 +229,10 @@ const char* lookme_kernel_name(int32_t kernel);
  * re-initialises the part it uses, so calls that may overlap on the GPU (on
  * different streams, or from different tables on the same device) race and
  * must be serialised by the caller.
- * Errors: INVALID_ARG, STATE (a scene not loaded yet), CUDA. */
+ * Errors: INVALID_ARG, STATE (a scene not loaded yet), CUDA.  A bounded
+ * device-side wait that gave up is not a return code of this call (it
+ * happens after the call returns): it sets the table's status word, read with
+ * lookme_device_status, and the tokens it left unrouted get scene -1. */
 #define LOOKME_ROUTE_STATIC_MAX_TOKENS 65536
 lookme_status lookme_route_scenes_static(lookme_table* table, const void* queries, int64_t n_tokens,
                                          int32_t* scene_out, lookme_stream stream);

@@ -999,10 +999,15 @@ lookme_status static_scratch(int device, StaticScratch* out) {
     return LOOKME_OK;
 }
 
+// A token whose key is still 0 was never scored (the routing kernel gave up a
+// bounded wait and set the status word): it gets scene -1, never a valid id.
 __global__ void k_route_static_decode(const unsigned long long* __restrict__ best, int64_t N, int64_t S,
                                       int32_t* __restrict__ scene_out) {
     const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (t < N) scene_out[t] = unpack_scene(best[t], S);
+    if (t < N) {
+        const unsigned long long k = best[t];
+        scene_out[t] = k == 0ull ? -1 : unpack_scene(k, S);
+    }
 }
 
 }  // namespace
@@ -1027,10 +1032,18 @@ extern "C" lookme_status lookme_route_scenes_static(lookme_table* t, const void*
     LaunchCtx ctx{s, t->num_sms};
     const int dk = (int)d.d_key;
     const float* bias = t->has_bias ? t->bias : nullptr;
-    // The prep kernel rewrites every key the routing kernel reduces into, so
-    // leftovers of an earlier call never leak into this one.
-    st = launch(t, s, KID_PREP, [&] { return launch_prep(ctx, d.dtype, queries, N, dk, sc.qnorm, nullptr, sc.best); });
-    if (st != LOOKME_OK) return st;
+    // Every key the routing kernel reduces into starts at 0, so leftovers of an
+    // earlier call never leak into this one: cleared by a memset (allocates
+    // nothing) before the tensor-core kernel, which computes the query norms
+    // itself, or by the prep kernel, which also computes them, before the
+    // CUDA-core one.
+    if (t->tc_route) {
+        cudaError_t e = cudaMemsetAsync(sc.best, 0, (size_t)N * sizeof(unsigned long long), s);
+        if (e != cudaSuccess) return cuda_fail(t, e, "clear routing keys");
+    } else {
+        st = launch(t, s, KID_PREP, [&] { return launch_prep(ctx, d.dtype, queries, N, dk, sc.qnorm, nullptr, sc.best); });
+        if (st != LOOKME_OK) return st;
+    }
     if (t->tc_route) {
         CUtensorMap mq;
         if (!encode_bf16_2d(&mq, queries, N, dk, 128))
