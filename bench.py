@@ -7,12 +7,18 @@ synthetic tokens: the single-image workload
 (1,024 tokens, d_k 256, 1,024 scenes x 256 primitives, d_v 2,048, bf16, top-8,
 keep 25%) unless --workload says otherwise.
 
-  value      tokens/s over K device-timed steps (CUDA events on the launching
-             stream; the step replayed as one CUDA graph of the library's
-             kernels; L2 flushed by writing then reading 512 MiB before every
-             step, outside the events), inputs resident in HBM.  The eager
-             time (the same calls issued one by one from Python) is reported
-             beside it.
+  value      tokens/s over K device-timed steps, inputs resident in HBM.  When
+             the table is small enough to hold several copies (single image:
+             10 replicas, 11.3 GiB), step i runs on replica i % R and the steps
+             alternate over two streams, so two batches are in flight (one
+             batch's routing and bucketing beside the other's level 2); the
+             steps are replayed as CUDA graphs of 64 steps between one pair of
+             events, and R - 1 other steps pass between two uses of a replica,
+             so its data is out of L2 (inputs larger than L2, no flush).
+             Otherwise one step per graph replay with L2 flushed by writing
+             then reading 512 MiB before every step, outside its events.
+             Reported beside it: the latency of one call at a time (L2
+             flushed, one graph replay) and the eager time.
   e2e        the same through host buffers: pinned-host queries and hidden
              states copied in and the updated hidden states copied out, inside
              the timed region
@@ -173,6 +179,41 @@ def aggregate_ranks(total_ms, e2e_ms, ws, n_tokens, steps, device):
     return total_ms, e2e_ms, value, e2e_value
 
 
+L2_BYTES = 129 << 20
+REPLICA_BUDGET = 24 << 30  # device bytes the table replicas may take
+MAX_REPLICAS = 16
+PIPE_STREAMS = 2           # batches in flight
+GRAPH_STEPS = 64           # steps per captured graph in the timed region
+
+
+def table_bytes(w):
+    S, P, e = w.n_scenes, w.n_prims, w.elem_bytes
+    return S * P * (w.d_key + w.d_value) * e + S * w.d_key * e
+
+
+def plan_replicas(w):
+    """How many table replicas the timed steps rotate through.
+
+    Each step reads about step_bytes that the previous steps did not; with R
+    replicas used in turn, R - 1 other steps (at least 5x L2 of traffic) pass
+    between two uses of one replica, so every step starts with its table data
+    out of L2 and no flush is needed.  R is a multiple of the stream count so
+    a replica always runs on the same stream.  Returns 1 (flush before every
+    step instead) when that many replicas do not fit the budget or the table
+    is not HBM-resident."""
+    from paper_2607_16305_gb300 import workloads as W
+
+    if w.residency != "device" or w.n_tables != 1:
+        return 1
+    d = W.expected_distinct(w.n_tokens, w.n_scenes)
+    step = algorithmic_bytes(w, d, int(w.n_tokens * w.keep_ratio))["step"]
+    need = 1 + math.ceil(5 * L2_BYTES / step)
+    need = ((need + PIPE_STREAMS - 1) // PIPE_STREAMS) * PIPE_STREAMS
+    if need > MAX_REPLICAS or need * table_bytes(w) > REPLICA_BUDGET:
+        return 1
+    return need
+
+
 def run_lookme(args, w, ws, rank, local):
     import torch
 
@@ -190,28 +231,33 @@ def run_lookme(args, w, ws, rank, local):
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
 
-    t = lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=w.dtype, device=local,
-                     max_tokens=w.n_tokens)
+    R = plan_replicas(w)
+    tabs = [lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=w.dtype, device=local,
+                         max_tokens=w.n_tokens) for _ in range(R)]
     cent = W.centroids(w, 0, dev)
     for c in range(w.n_chunks):
         k, v = W.table_chunk(w, 0, c, dev, None, cent)
         s0 = c * w.scenes_per_chunk
-        t.load_scenes(s0, k, v, centroids=cent[s0:s0 + k.shape[0]])
+        for t in tabs:  # every replica holds the same table
+            t.load_scenes(s0, k, v, centroids=cent[s0:s0 + k.shape[0]])
         del k, v
-    q = W.queries(w, dev)
-    hidden = [W.hidden(w, l, dev) for l in range(w.layers_per_table)]
-    N, K = w.n_tokens, w.top_k
-    scene = torch.empty(N, dtype=torch.int32, device=dev)
-    prim = torch.empty(N, K, dtype=torch.int32, device=dev)
-    weight = torch.empty(N, K, dtype=torch.float32, device=dev)
-    mask = torch.empty(N, dtype=torch.uint8, device=dev)
+    q0 = W.queries(w, dev)
+    N, K, L = w.n_tokens, w.top_k, w.layers_per_table
+    # Per replica: its own queries, hidden states and outputs.
+    qs = [q0 if r == 0 else q0.clone() for r in range(R)]
+    hs = [[W.hidden(w, l, dev) for l in range(L)] for _ in range(R)]
+    outs = [(torch.empty(N, dtype=torch.int32, device=dev), torch.empty(N, K, dtype=torch.int32, device=dev),
+             torch.empty(N, K, dtype=torch.float32, device=dev), torch.empty(N, dtype=torch.uint8, device=dev))
+            for _ in range(R)]
     seg = w.segment_offsets if w.n_segments > 1 else None
     flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
     flush_sink = torch.zeros((), dtype=torch.int64, device=dev)
+    streams = [torch.cuda.Stream(dev) for _ in range(PIPE_STREAMS)] if R > 1 else [stream]
 
-    def step():
-        t.lookup_inject(q, K, hidden, w.keep_ratio, seg_offsets=seg, scene_out=scene, prim_out=prim,
-                        weight_out=weight, mask_out=mask)
+    def step(r, q=None, hidden=None):
+        sc, pr, wt, mk = outs[r]
+        tabs[r].lookup_inject(qs[r] if q is None else q, K, hs[r] if hidden is None else hidden, w.keep_ratio,
+                              seg_offsets=seg, scene_out=sc, prim_out=pr, weight_out=wt, mask_out=mk)
 
     def flush_l2(i):
         # Write then read a buffer four times L2's size: the step starts with no
@@ -219,76 +265,139 @@ def run_lookme(args, w, ws, rank, local):
         flush.fill_(i & 0xFF)
         flush_sink.copy_(flush.sum(dtype=torch.int64))
 
-    for _ in range(args.warmup):
-        flush_l2(1)
-        step()
-    torch.cuda.synchronize(dev)
-    stats = t.stats()
-    n_sel = int(mask.sum().item())
+    def pipelined(n, body):
+        # Step i on replica i % R, issued on stream i % PIPE_STREAMS: two
+        # batches in flight, each replica always on the same stream.
+        cur = torch.cuda.current_stream(dev)
+        for s in streams:
+            s.wait_stream(cur)
+        for i in range(n):
+            with torch.cuda.stream(streams[i % len(streams)]):
+                body(i % R)
+        for s in streams:
+            cur.wait_stream(s)
 
-    # The step as one CUDA graph (the library never allocates or syncs inside a
-    # call once scratch is reserved), replayed per timed step.
-    graph = torch.cuda.CUDAGraph()
+    for i in range(args.warmup):
+        if R == 1:
+            flush_l2(1)
+        step(i % R)
+    torch.cuda.synchronize(dev)
+    stats = tabs[0].stats()
+    n_sel = int(outs[0][3].sum().item())
+    c0 = tabs[0].launch_count()
+    step(0)
+    torch.cuda.synchronize(dev)
+    launches_per_step = tabs[0].launch_count() - c0
+
+    # Graphs of the steps (the library never allocates or syncs inside a call
+    # once scratch is reserved).  With replicas: up to GRAPH_STEPS steps per
+    # graph, pipelined over the streams; without: one step per graph.
     side = torch.cuda.Stream(dev)
     side.wait_stream(stream)
     with torch.cuda.stream(side):
-        step()
+        for r in range(R):
+            step(r)
     stream.wait_stream(side)
-    with torch.cuda.graph(graph):
-        step()
     torch.cuda.synchronize(dev)
 
-    c0 = t.launch_count()
-    step()
+    def capture(n):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            if R > 1:
+                pipelined(n, step)
+            else:
+                step(0)
+        return g
+
+    g1 = capture(1) if R == 1 else None
+    if R > 1:
+        per_graph = min(args.steps, GRAPH_STEPS)
+        g_full = capture(per_graph)
+        rem = args.steps % per_graph
+        g_rem = capture(rem) if rem else None
     torch.cuda.synchronize(dev)
-    launches_per_step = t.launch_count() - c0
 
     sampler = ClockSampler(local)
     sampler.start()
     # ---------------------------------------------------------- timed: value
-    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     if ws > 1:
         import torch.distributed as dist
 
         dist.barrier()
     torch.cuda.synchronize(dev)
-    for i in range(args.steps):
-        flush_l2(i)
-        starts[i].record(stream)
-        graph.replay()
-        ends[i].record(stream)
-    torch.cuda.synchronize(dev)
+    if R > 1:
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        for _ in range(args.steps // per_graph):
+            g_full.replay()
+        if g_rem is not None:
+            g_rem.replay()
+        ev1.record(stream)
+        torch.cuda.synchronize(dev)
+        total_ms = ev0.elapsed_time(ev1)
+    else:
+        starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        for i in range(args.steps):
+            flush_l2(i)
+            starts[i].record(stream)
+            g1.replay()
+            ends[i].record(stream)
+        torch.cuda.synchronize(dev)
+        total_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends))
     if ws > 1:
         dist.barrier()
-    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    total_ms = sum(step_ms)
     launches = launches_per_step * args.steps
 
-    # ------------------------------------ the same steps as eager C-ABI calls
-    estarts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    eends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    # -------------- one call at a time: L2 flushed, one graph replay per call
+    if g1 is None:
+        g1 = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g1):
+            step(0)
+        torch.cuda.synchronize(dev)
+    lstarts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    lends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     for i in range(args.steps):
         flush_l2(i)
-        estarts[i].record(stream)
-        step()
-        eends[i].record(stream)
+        lstarts[i].record(stream)
+        g1.replay()
+        lends[i].record(stream)
     torch.cuda.synchronize(dev)
-    eager_ms = sum(s.elapsed_time(e) for s, e in zip(estarts, eends)) / args.steps
+    latency_ms = sum(s.elapsed_time(e) for s, e in zip(lstarts, lends)) / args.steps
+
+    # ---------------------- the same steps as eager C-ABI calls from Python
+    if R > 1:
+        ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ea.record(stream)
+        pipelined(args.steps, step)
+        eb.record(stream)
+        torch.cuda.synchronize(dev)
+        eager_ms = ea.elapsed_time(eb) / args.steps
+    else:
+        estarts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        eends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        for i in range(args.steps):
+            flush_l2(i)
+            estarts[i].record(stream)
+            step(0)
+            eends[i].record(stream)
+        torch.cuda.synchronize(dev)
+        eager_ms = sum(s.elapsed_time(e) for s, e in zip(estarts, eends)) / args.steps
 
     # ----------------------------------------- per-kernel durations (traced)
-    t.trace_enable(True)
-    t.trace_read()
+    t0 = tabs[0]
+    t0.trace_enable(True)
+    t0.trace_read()
     tstarts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     tends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     for i in range(args.steps):
         flush_l2(i)
         tstarts[i].record(stream)
-        step()
+        step(0)
         tends[i].record(stream)
     torch.cuda.synchronize(dev)
-    recs = t.trace_read(max_records=args.steps * 8 + 16)
-    t.trace_enable(False)
+    recs = t0.trace_read(max_records=args.steps * 8 + 16)
+    t0.trace_enable(False)
     traced_ms = sum(s.elapsed_time(e) for s, e in zip(tstarts, tends))
     per_kernel = {}
     for name, ms in recs:
@@ -296,33 +405,47 @@ def run_lookme(args, w, ws, rank, local):
     kernels_ms = {k: statistics.mean(v) for k, v in per_kernel.items()}
 
     # ------------------------------------------------- e2e through host buffers
-    q_host = q.cpu().pin_memory()
-    h_host = [h.cpu().pin_memory() for h in hidden]
-    h_out = [torch.empty_like(h).pin_memory() for h in h_host]
-    q_dev = torch.empty_like(q)
-    h_dev = [torch.empty_like(h) for h in hidden]
-    e_starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    e_ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    for i in range(args.steps):
-        flush_l2(i)
-        e_starts[i].record(stream)
-        q_dev.copy_(q_host, non_blocking=True)
-        for hd, hh in zip(h_dev, h_host):
+    # Every step copies its queries and hidden states in from pinned host
+    # memory and the updated hidden states back, on the step's stream.
+    q_host = [qs[r].cpu().pin_memory() for r in range(R)]
+    h_host = [[h.cpu().pin_memory() for h in hs[r]] for r in range(R)]
+    h_out = [[torch.empty_like(h).pin_memory() for h in h_host[r]] for r in range(R)]
+    q_dev = [torch.empty_like(q0) for _ in range(R)]
+    h_dev = [[torch.empty_like(h) for h in hs[r]] for r in range(R)]
+
+    def e2e_step(r):
+        q_dev[r].copy_(q_host[r], non_blocking=True)
+        for hd, hh in zip(h_dev[r], h_host[r]):
             hd.copy_(hh, non_blocking=True)
-        t.lookup_inject(q_dev, K, h_dev, w.keep_ratio, seg_offsets=seg, scene_out=scene, prim_out=prim,
-                        weight_out=weight, mask_out=mask)
-        for ho, hd in zip(h_out, h_dev):
+        step(r, q=q_dev[r], hidden=h_dev[r])
+        for ho, hd in zip(h_out[r], h_dev[r]):
             ho.copy_(hd, non_blocking=True)
-        e_ends[i].record(stream)
-    torch.cuda.synchronize(dev)
-    e2e_ms = sum(s.elapsed_time(e) for s, e in zip(e_starts, e_ends))
+
+    if R > 1:
+        xa, xb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        xa.record(stream)
+        pipelined(args.steps, e2e_step)
+        xb.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = xa.elapsed_time(xb)
+    else:
+        e_starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        e_ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        for i in range(args.steps):
+            flush_l2(i)
+            e_starts[i].record(stream)
+            e2e_step(0)
+            e_ends[i].record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = sum(s.elapsed_time(e) for s, e in zip(e_starts, e_ends))
     clocks = sampler.stop()
-    assert t.device_status() == 0, "a device-side wait timed out"
+    for t in tabs:
+        assert t.device_status() == 0, "a device-side wait timed out"
 
     total_ms, e2e_ms, value, e2e_value = aggregate_ranks(total_ms, e2e_ms, ws, N, args.steps, dev)
 
-    h2d = q.numel() * q.element_size() + sum(h.numel() * h.element_size() for h in hidden)
-    d2h = sum(h.numel() * h.element_size() for h in hidden)
+    h2d = q0.numel() * q0.element_size() + sum(h.numel() * h.element_size() for h in hs[0])
+    d2h = sum(h.numel() * h.element_size() for h in hs[0])
     ms_per_step = total_ms / args.steps
 
     peaks, peak_kind = load_peaks()
@@ -331,14 +454,21 @@ def run_lookme(args, w, ws, rank, local):
     score_ms = kernels_ms.get("score")
     achieved = ab["score"] / (score_ms * 1e-3) / 1e9 if score_ms else None
     step_gbs = ab["step"] / (ms_per_step * 1e-3) / 1e9
+    if R > 1:
+        l2 = (f"inputs larger than L2: {R} replicas of the table ({table_bytes(w) * R / 2**30:.1f} GiB) used in turn, "
+              f"{R - 1} other steps between two uses of one replica; no flush")
+        launch = (f"{PIPE_STREAMS} batches in flight: step i on replica i % {R} on stream i % {PIPE_STREAMS}; "
+                  f"{per_graph} steps per CUDA graph; one event pair around all {args.steps} steps")
+    else:
+        l2 = f"flushed before every step ({FLUSH_BYTES >> 20} MiB written then read, outside the events)"
+        launch = "step replayed as one CUDA graph (kernels chained by programmatic dependent launch)"
     result = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": w.dtype, "data": "synthetic (seeded Gaussian mixture, random tables)",
         "config": {"workload": w.name, "tokens": N, "d_key": w.d_key, "scenes": w.n_scenes, "prims": w.n_prims,
-                   "d_value": w.d_value, "top_k": K, "keep_ratio": w.keep_ratio, "layers": w.layers_per_table,
-                   "l2": f"flushed before every step ({FLUSH_BYTES >> 20} MiB written then read, outside the events)",
-                   "launch": "step replayed as one CUDA graph (kernels chained by programmatic dependent launch)",
+                   "d_value": w.d_value, "top_k": K, "keep_ratio": w.keep_ratio, "layers": L,
+                   "replicas": R, "l2": l2, "launch": launch,
                    "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "kernel": "score (level-2 key scoring + top-k + softmax)",
                      "achieved": achieved, "peak": hbm, "unit": "GB/s",
@@ -346,7 +476,10 @@ def run_lookme(args, w, ws, rank, local):
                      "algorithmic_bytes": ab["score"], "mean_ms": score_ms,
                      "traffic": profiled_traffic("score", w.name)},
         "step_roofline": {"bound": "hbm", "algorithmic_bytes": ab["step"], "achieved": step_gbs, "peak": hbm,
-                          "unit": "GB/s", "frac": step_gbs / hbm, "roofline_us": ab["step"] / hbm / 1e3},
+                          "unit": "GB/s", "frac": step_gbs / hbm, "roofline_us": ab["step"] / hbm / 1e3,
+                          "peak_source": peak_kind},
+        "latency_ms_per_call": latency_ms,
+        "latency_method": "one call at a time: L2 flushed before each, one CUDA-graph replay, events around it",
         "eager_ms_per_step": eager_ms,
         "kernels_ms": kernels_ms, "traced_ms_per_step": traced_ms / args.steps,
         "routed_scenes": stats["n_routed_scenes"], "selected_tokens": n_sel,
@@ -355,7 +488,8 @@ def run_lookme(args, w, ws, rank, local):
         "gpu_launches": launches,
         "clocks": clocks,
     }
-    t.close()
+    for t in tabs:
+        t.close()
     return result
 
 
