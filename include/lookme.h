@@ -79,7 +79,9 @@ typedef struct {
     int32_t device;       /* CUDA device ordinal */
     int32_t reserved0;    /* must be 0 */
     int64_t max_tokens;   /* scratch is sized for this many tokens per call; 0 = grow on demand */
-    int64_t stage_slots;  /* HOST_STAGED: scenes the HBM slot cache holds (0 = n_scenes) */
+    int64_t stage_slots;  /* HOST_STAGED: scenes the HBM slot cache holds (0 = n_scenes); a call
+                           * may route to at most this many distinct scenes, so it must be at
+                           * least min(n_tokens, n_scenes) of every lookup */
 } lookme_table_desc;
 
 typedef struct lookme_table lookme_table; /* opaque, owned by the library */
@@ -130,8 +132,17 @@ lookme_status lookme_load_scenes(lookme_table* table, int64_t scene_begin, int64
  *   qnorm_out   device [n_tokens] fp32 ||q_t||_2, or NULL (the table keeps
  *               its own copy for lookme_inject's default priority)
  * Every token is looked up; selection happens in lookme_inject.
+ * HOST_STAGED tables (Sec. "Level-2: scene-primitive retrieval", last
+ * sentence: scene blocks are loaded on demand): after bucketing, the routed
+ * scenes are looked up in the table's HBM slot cache, which persists across
+ * calls; the key blocks of the misses are copied from pinned host memory over
+ * the host link on the table's own staging stream (forked from and joined to
+ * the caller's stream with events), evicting scenes that this call does not
+ * route to (clock order); level 2 then reads the slots, and the injection
+ * reads the selected value rows from host memory directly.
  * Errors: INVALID_ARG, STATE (a scene not loaded yet, or scratch would have to
- * grow while the stream is being captured), OOM, CUDA. */
+ * grow while the stream is being captured), UNSUPPORTED (HOST_STAGED with
+ * fewer staging slots than min(n_tokens, n_scenes)), OOM, CUDA. */
 lookme_status lookme_lookup(lookme_table* table, const void* queries, int64_t n_tokens, int32_t top_k,
                             int32_t* scene_out, int32_t* prim_out, float* weight_out, float* qnorm_out,
                             lookme_stream stream);
@@ -180,13 +191,22 @@ lookme_status lookme_lookup_inject(lookme_table* table, const void* queries, int
  * calls (for example under CUDA graph capture) never allocate.  Synchronous. */
 lookme_status lookme_reserve(lookme_table* table, int64_t max_tokens);
 
+/* Empty the HOST_STAGED slot cache, so that the next lookup copies every
+ * routed scene's key block again (for cold-cache measurements, or after the
+ * host copy of the table was changed other than through lookme_load_scenes,
+ * which empties the cache itself).  Asynchronous on the stream; no effect on
+ * HBM-resident tables.  Errors: INVALID_ARG, CUDA. */
+lookme_status lookme_stage_invalidate(lookme_table* table, lookme_stream stream);
+
 /* Statistics of the table's most recent lookup, read back synchronously on
  * the given stream: routed scenes, level-2 work items, largest bucket. */
 typedef struct {
     int64_t n_tokens;
     int32_t n_routed_scenes;  /* distinct scenes that received a token */
     int32_t n_work_items;     /* level-2 work items (scene, token chunk) */
-    int64_t staged_bytes;     /* HOST_STAGED: key bytes copied host -> HBM */
+    int64_t staged_bytes;     /* HOST_STAGED: key bytes copied host -> HBM (the slot cache's misses) */
+    int32_t staged_hits;      /* HOST_STAGED: routed scenes found in the slot cache */
+    int32_t reserved0;
 } lookme_lookup_stats;
 lookme_status lookme_last_lookup_stats(lookme_table* table, lookme_lookup_stats* out, lookme_stream stream);
 

@@ -31,6 +31,7 @@ enum KernelId : int32_t {
     KID_BUCKET_SCAN = 14,     // K2 for large calls: work list from the counts
     KID_BUCKET_SCATTER = 15,  // K2 for large calls: token ids into their items
     KID_STEP = 16,            // K1 + K2 + K3 (+ gate and K4): the fused step on tcgen05
+    KID_STAGE_ASSIGN = 17,    // K6a: slot cache look-up and the copy list
     KID_COUNT
 };
 
@@ -39,6 +40,7 @@ constexpr uint32_t STATUS_WAIT_TIMEOUT = 1u;
 constexpr uint32_t STATUS_IN_ROUTE = 2u;  // set with STATUS_WAIT_TIMEOUT by the level-1 kernel
 constexpr uint32_t STATUS_IN_SCORE = 4u;  // set with STATUS_WAIT_TIMEOUT by a level-2 kernel
 constexpr uint32_t STATUS_IN_STEP = 8u;   // set with STATUS_WAIT_TIMEOUT by the fused step kernel
+constexpr uint32_t STATUS_STAGE_OVERFLOW = 16u;  // more routed scenes than HBM slots (keys not staged)
 
 // ------------------------------------------------------------ element access
 __device__ __forceinline__ float to_f32(float x) { return x; }
@@ -263,9 +265,32 @@ cudaError_t launch_inject_records(const LaunchCtx& c, const InjectArgs& a, const
 constexpr int64_t kFusedMaxSegment = 8192;
 cudaError_t launch_select_inject(const LaunchCtx& c, const InjectArgs& a, const float* priority,
                                  const int64_t* seg_off_host, int n_seg, double keep_ratio, uint8_t* mask);
-// K6
+// K6: the HBM slot cache of a pinned-host table, kept across calls.  Per
+// scene its slot or -1 (slot_of), per slot its scene or -1 (slot_scene) and
+// the number of the last call that used it (slot_stamp), and this header.
+struct StageCache {
+    int32_t epoch;     // calls so far (stamps the slots each call uses)
+    int32_t hand;      // where the next search for free slots starts
+    int32_t n_copy;    // key blocks the last call copied from the host
+    int32_t n_hit;     // routed scenes the last call found in HBM
+};
+struct StageArgs {
+    int32_t* slot_of;     // [S]
+    int32_t* slot_scene;  // [n_slots]
+    int32_t* slot_stamp;  // [n_slots]
+    int32_t* route_slot;  // [S] per routed-list index: its slot (scratch)
+    int32_t* copy_slot;   // [n_slots] copies of this call: slot and scene
+    int32_t* copy_scene;  // [n_slots]
+    StageCache* hdr;
+    int64_t n_slots;
+};
+// K6a (one CTA): find each routed scene's slot, give the misses free or
+// least-recently-reached slots, list the copies, point the work items at
+// their slots.  K6b: copy the listed key blocks over the host mapping.
+cudaError_t launch_stage_assign(const LaunchCtx& c, const StageArgs& sa, const int32_t* routed,
+                                const int32_t* counters, WorkItem* work, uint32_t* status);
 cudaError_t launch_stage(const LaunchCtx& c, const void* keys_host_mapped, void* slots, int64_t block_bytes,
-                         int64_t n_slots, const int32_t* routed, const int32_t* counters);
+                         const StageArgs& sa);
 
 // ------------------------------------------------------------- fused step
 // Routing, bucketing, level 2, the injection gate and the injection in one

@@ -42,7 +42,7 @@ const char* kKernelNames[KID_COUNT] = {"prep",         "route_tc", "route_simt",
                                        "score",        "select",   "inject",        "stage",
                                        "centroid_mean", "inv_cnorm", "route_decode", "select_inject",
                                        "tile_keys",    "bucket_count", "bucket_scan", "bucket_scatter",
-                                       "step"};
+                                       "step",         "stage_assign"};
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point, so the
 // library does not link libcuda directly.
@@ -114,6 +114,10 @@ struct lookme_table {
     void* values_host = nullptr;
     void* slots = nullptr;      // HBM slot cache of staged key blocks
     int64_t n_slots = 0;
+    StageArgs stage{};          // the slot cache's map (device), kept across calls
+    void* stage_mem = nullptr;
+    cudaStream_t stage_stream = nullptr;  // the copies run here, ordered by events
+    cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
     void* cent = nullptr;
     float* inv_cnorm = nullptr;
     float* bias = nullptr;
@@ -285,6 +289,10 @@ void destroy_table(lookme_table* t) {
         if (t->keys_host) cudaFreeHost(t->keys_host);
         if (t->values_host) cudaFreeHost(t->values_host);
         if (t->slots) cudaFree(t->slots);
+        if (t->stage_mem) cudaFree(t->stage_mem);
+        if (t->ev_fork) cudaEventDestroy(t->ev_fork);
+        if (t->ev_join) cudaEventDestroy(t->ev_join);
+        if (t->stage_stream) cudaStreamDestroy(t->stage_stream);
     }
     if (t->cent) cudaFree(t->cent);
     if (t->inv_cnorm) cudaFree(t->inv_cnorm);
@@ -392,8 +400,29 @@ lookme_status lookme_table_create(const lookme_table_desc* desc, lookme_table** 
              cudaHostAlloc(&t->values_host, vbytes, cudaHostAllocMapped | cudaHostAllocPortable) == cudaSuccess &&
              cudaHostGetDevicePointer(&t->keys, t->keys_host, 0) == cudaSuccess &&
              cudaHostGetDevicePointer(&t->values, t->values_host, 0) == cudaSuccess;
-        t->n_slots = d.stage_slots > 0 ? d.stage_slots : d.n_scenes;
+        t->n_slots = d.stage_slots > 0 ? std::min<int64_t>(d.stage_slots, d.n_scenes) : d.n_scenes;
         ok = ok && cudaMalloc(&t->slots, (size_t)t->n_slots * t->kblock) == cudaSuccess;
+        // The slot cache's map: slot_of and route_slot [S], slot_scene,
+        // slot_stamp, copy_slot and copy_scene [n_slots], the header.
+        const size_t a = align_up(S * sizeof(int32_t), 256), b = align_up(t->n_slots * sizeof(int32_t), 256);
+        ok = ok && cudaMalloc(&t->stage_mem, 2 * a + 4 * b + 256) == cudaSuccess &&
+             cudaStreamCreateWithFlags(&t->stage_stream, cudaStreamNonBlocking) == cudaSuccess &&
+             cudaEventCreateWithFlags(&t->ev_fork, cudaEventDisableTiming) == cudaSuccess &&
+             cudaEventCreateWithFlags(&t->ev_join, cudaEventDisableTiming) == cudaSuccess;
+        if (ok) {
+            char* m = static_cast<char*>(t->stage_mem);
+            t->stage.slot_of = reinterpret_cast<int32_t*>(m);
+            t->stage.route_slot = reinterpret_cast<int32_t*>(m + a);
+            t->stage.slot_scene = reinterpret_cast<int32_t*>(m + 2 * a);
+            t->stage.slot_stamp = reinterpret_cast<int32_t*>(m + 2 * a + b);
+            t->stage.copy_slot = reinterpret_cast<int32_t*>(m + 2 * a + 2 * b);
+            t->stage.copy_scene = reinterpret_cast<int32_t*>(m + 2 * a + 3 * b);
+            t->stage.hdr = reinterpret_cast<StageCache*>(m + 2 * a + 4 * b);
+            t->stage.n_slots = t->n_slots;
+            ok = cudaMemset(t->stage_mem, 0, 2 * a + 4 * b + 256) == cudaSuccess &&
+                 cudaMemset(t->stage.slot_of, 0xFF, S * sizeof(int32_t)) == cudaSuccess &&
+                 cudaMemset(t->stage.slot_scene, 0xFF, t->n_slots * sizeof(int32_t)) == cudaSuccess;
+        }
     }
     ok = ok && cudaMalloc(&t->cent, align_up(S * d.d_key * t->esz, 256)) == cudaSuccess &&
          cudaMalloc(&t->inv_cnorm, align_up(S * sizeof(float), 256)) == cudaSuccess &&
@@ -447,6 +476,26 @@ lookme_status lookme_reserve(lookme_table* t, int64_t max_tokens) {
     if (max_tokens < 0) return fail(LOOKME_ERR_INVALID_ARG, "max_tokens < 0");
     DeviceGuard guard(t->d.device);
     return ensure_scratch(t, max_tokens, nullptr);
+}
+
+// Forgets what the HBM slot cache holds (asynchronous, on stream s).
+cudaError_t stage_invalidate(lookme_table* t, cudaStream_t s) {
+    const StageArgs& g = t->stage;
+    cudaError_t e = cudaMemsetAsync(g.slot_of, 0xFF, t->d.n_scenes * sizeof(int32_t), s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(g.slot_scene, 0xFF, t->n_slots * sizeof(int32_t), s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(g.slot_stamp, 0, t->n_slots * sizeof(int32_t), s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(g.hdr, 0, sizeof(StageCache), s);
+    return e;
+}
+
+lookme_status lookme_stage_invalidate(lookme_table* t, lookme_stream stream) {
+    lookme_status st = check_table(t);
+    if (st != LOOKME_OK) return st;
+    if (t->d.residency != LOOKME_RES_HOST_STAGED) return LOOKME_OK;
+    DeviceGuard guard(t->d.device);
+    cudaError_t e = stage_invalidate(t, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(t, e, "slot cache reset");
+    return LOOKME_OK;
 }
 
 lookme_status lookme_load_scenes(lookme_table* t, int64_t scene_begin, int64_t n, const void* centroids,
@@ -510,6 +559,10 @@ lookme_status lookme_load_scenes(lookme_table* t, int64_t scene_begin, int64_t n
             return cuda_fail(t, e, "copy bias");
         t->has_bias = true;
     }
+    // Cached key blocks of reloaded scenes would be stale: start the slot
+    // cache afresh.
+    if (d.residency == LOOKME_RES_HOST_STAGED && (e = stage_invalidate(t, s)) != cudaSuccess)
+        return cuda_fail(t, e, "slot cache reset");
     for (int64_t i = scene_begin; i < scene_begin + n; ++i) {
         if (!t->loaded[i]) {
             t->loaded[i] = 1;
@@ -536,7 +589,7 @@ lookme_status check_lookup(const lookme_table* t, const void* queries, int64_t N
     if (t->n_loaded != d.n_scenes)
         return fail(LOOKME_ERR_STATE, "%lld of %lld scenes loaded", (long long)t->n_loaded, (long long)d.n_scenes);
     if (d.residency == LOOKME_RES_HOST_STAGED && std::min<int64_t>(N, d.n_scenes) > t->n_slots)
-        return fail(LOOKME_ERR_UNSUPPORTED, "up to %lld routed scenes but only %lld staging slots",
+        return fail(LOOKME_ERR_UNSUPPORTED, "up to %lld routed scenes in one call but only %lld staging slots",
                     (long long)std::min<int64_t>(N, d.n_scenes), (long long)t->n_slots);
     return LOOKME_OK;
 }
@@ -677,10 +730,24 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
     if (st != LOOKME_OK) return st;
     const bool staged = d.residency == LOOKME_RES_HOST_STAGED;
     if (staged) {
-        st = launch(t, s, KID_STAGE, [&] {
-            return launch_stage(ctx, t->keys, t->slots, t->kblock, t->n_slots, t->routed, t->counters);
+        // Slot look-up on the caller's stream; the copies of the misses on the
+        // table's staging stream, forked after the look-up and joined before
+        // level 2 (the next call's copies therefore start only after this
+        // call's level 2, which reads the slots, is done).
+        st = launch(t, s, KID_STAGE_ASSIGN, [&] {
+            return launch_stage_assign(ctx, t->stage, t->routed, t->counters, t->work, t->status);
         });
         if (st != LOOKME_OK) return st;
+        cudaError_t e = cudaEventRecord(t->ev_fork, s);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(t->stage_stream, t->ev_fork, 0);
+        if (e != cudaSuccess) return cuda_fail(t, e, "staging fork");
+        LaunchCtx sctx{t->stage_stream, t->num_sms};
+        st = launch(t, t->stage_stream, KID_STAGE,
+                    [&] { return launch_stage(sctx, t->keys, t->slots, t->kblock, t->stage); });
+        if (st != LOOKME_OK) return st;
+        e = cudaEventRecord(t->ev_join, t->stage_stream);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(s, t->ev_join, 0);
+        if (e != cudaSuccess) return cuda_fail(t, e, "staging join");
     }
     ScoreArgs a;
     a.dtype = d.dtype;
@@ -896,16 +963,18 @@ lookme_status lookme_last_lookup_stats(lookme_table* t, lookme_lookup_stats* out
     if (t->last_tokens < 0 || !t->counters) return LOOKME_OK;
     DeviceGuard guard(t->d.device);
     int32_t c[4];
+    StageCache hc{};
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = cudaMemcpyAsync(c, t->counters, sizeof(c), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess && t->d.residency == LOOKME_RES_HOST_STAGED)
+        e = cudaMemcpyAsync(&hc, t->stage.hdr, sizeof(hc), cudaMemcpyDeviceToHost, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(t, e, "read lookup stats");
     out->n_tokens = t->last_tokens;
     out->n_work_items = c[0];
     out->n_routed_scenes = c[1];
-    out->staged_bytes = t->d.residency == LOOKME_RES_HOST_STAGED
-                            ? (int64_t)c[1] * t->d.n_prims * t->d.d_key * (int64_t)t->esz
-                            : 0;
+    out->staged_bytes = (int64_t)hc.n_copy * t->kblock;
+    out->staged_hits = hc.n_hit;
     return LOOKME_OK;
 }
 

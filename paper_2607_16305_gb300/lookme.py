@@ -24,7 +24,7 @@ ROUTE_STATIC_MAX_TOKENS = 65536
 
 EXPORTS = [
     "lookme_table_create", "lookme_table_destroy", "lookme_load_scenes", "lookme_lookup", "lookme_inject",
-    "lookme_reserve", "lookme_last_lookup_stats", "lookme_device_status", "lookme_launch_count",
+    "lookme_reserve", "lookme_stage_invalidate", "lookme_last_lookup_stats", "lookme_device_status", "lookme_launch_count",
     "lookme_trace_enable", "lookme_trace_read", "lookme_kernel_name", "lookme_status_string",
     "lookme_last_error", "lookme_route_scenes_static", "lookme_lookup_inject",
 ]
@@ -47,7 +47,8 @@ class TableDesc(ctypes.Structure):
 
 class LookupStats(ctypes.Structure):
     _fields_ = [("n_tokens", ctypes.c_int64), ("n_routed_scenes", ctypes.c_int32),
-                ("n_work_items", ctypes.c_int32), ("staged_bytes", ctypes.c_int64)]
+                ("n_work_items", ctypes.c_int32), ("staged_bytes", ctypes.c_int64),
+                ("staged_hits", ctypes.c_int32), ("reserved0", ctypes.c_int32)]
 
 
 class TraceRecord(ctypes.Structure):
@@ -73,6 +74,7 @@ def load(path: str = LIB_PATH):
         "lookme_lookup": ([P, P, I64, I32, P, P, P, P, P], I32),
         "lookme_inject": ([P, P, P, P, I64, I32, P, P, I32, D, P, I32, P, P, P], I32),
         "lookme_reserve": ([P, I64], I32),
+        "lookme_stage_invalidate": ([P, P], I32),
         "lookme_last_lookup_stats": ([P, ctypes.POINTER(LookupStats), P], I32),
         "lookme_device_status": ([P, ctypes.POINTER(ctypes.c_uint32), I32, P], I32),
         "lookme_launch_count": ([P], ctypes.c_uint64),
@@ -238,7 +240,11 @@ class Table:
         s = LookupStats()
         _check(self.lib.lookme_last_lookup_stats(self.handle, ctypes.byref(s), _stream(stream, self.device)))
         return dict(n_tokens=s.n_tokens, n_routed_scenes=s.n_routed_scenes, n_work_items=s.n_work_items,
-                    staged_bytes=s.staged_bytes)
+                    staged_bytes=s.staged_bytes, staged_hits=s.staged_hits)
+
+    def stage_invalidate(self, stream=None):
+        """Empty the HBM slot cache of a pinned-host table (the next lookup copies every routed scene)."""
+        _check(self.lib.lookme_stage_invalidate(self.handle, _stream(stream, self.device)))
 
     def device_status(self, reset=False, stream=None):
         v = ctypes.c_uint32()
