@@ -493,6 +493,166 @@ def run_lookme(args, w, ws, rank, local):
     return result
 
 
+def run_multitable(args, w, ws, rank, local):
+    """Several tables over one query set (each table shared by layers_per_table
+    layers), tables in pinned host memory staged to HBM on demand.
+
+    A step = one lookme_lookup_inject per table, tables alternating over two
+    streams so that one table's routing, bucketing and key staging overlap the
+    previous table's level 2 and injection.  Cold: each table's slot cache is
+    emptied and L2 flushed before every step (outside the events), so every
+    routed scene's key block crosses the host link; warm: the caches persist
+    (the same queries every step, so every routed scene is a hit)."""
+    import torch
+
+    from __graft_entry__ import build
+    from paper_2607_16305_gb300 import lookme
+    from paper_2607_16305_gb300 import workloads as W
+
+    if rank == 0:
+        build()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    T, L, N, K = w.n_tables, w.layers_per_table, w.n_tokens, w.top_k
+    mu = W.means(w, dev)
+    tabs = []
+    for ti in range(T):
+        t = lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=w.dtype, residency="host",
+                         device=local, max_tokens=N)
+        cent = W.centroids(w, ti, dev, mu)
+        for c in range(w.n_chunks):
+            k, v = W.table_chunk(w, ti, c, dev, mu, cent)
+            s0 = c * w.scenes_per_chunk
+            t.load_scenes(s0, k, v, centroids=cent[s0:s0 + k.shape[0]])
+            del k, v
+        tabs.append(t)
+    q = W.queries(w, dev, mu)
+    hidden = [W.hidden(w, l, dev) for l in range(T * L)]
+    outs = [(torch.empty(N, dtype=torch.int32, device=dev), torch.empty(N, K, dtype=torch.int32, device=dev),
+             torch.empty(N, K, dtype=torch.float32, device=dev), torch.empty(N, dtype=torch.uint8, device=dev))
+            for _ in range(T)]
+    streams = [torch.cuda.Stream(dev) for _ in range(PIPE_STREAMS)]
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
+    flush_sink = torch.zeros((), dtype=torch.int64, device=dev)
+
+    def step():
+        cur = torch.cuda.current_stream(dev)
+        for s in streams:
+            s.wait_stream(cur)
+        for ti in range(T):
+            sc, pr, wt, mk = outs[ti]
+            with torch.cuda.stream(streams[ti % len(streams)]):
+                tabs[ti].lookup_inject(q, K, hidden[ti * L:(ti + 1) * L], w.keep_ratio, scene_out=sc, prim_out=pr,
+                                       weight_out=wt, mask_out=mk)
+        for s in streams:
+            cur.wait_stream(s)
+
+    def cold_prep(i):
+        for t in tabs:
+            t.stage_invalidate(stream)
+        flush.fill_(i & 0xFF)
+        flush_sink.copy_(flush.sum(dtype=torch.int64))
+
+    for i in range(args.warmup):
+        cold_prep(i)
+        step()
+    torch.cuda.synchronize(dev)
+    stats = [t.stats() for t in tabs]
+    staged = sum(s["staged_bytes"] for s in stats)
+    routed = [s["n_routed_scenes"] for s in stats]
+    n_sel = int(outs[0][3].sum().item())
+    c0 = sum(t.launch_count() for t in tabs)
+    step()
+    torch.cuda.synchronize(dev)
+    launches_per_step = sum(t.launch_count() for t in tabs) - c0
+
+    # Host link reference: one pinned-host -> HBM copy engine transfer.
+    hbuf = torch.empty(256 << 20, dtype=torch.uint8).pin_memory()
+    dbuf = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for _ in range(3):
+        dbuf.copy_(hbuf, non_blocking=True)
+    la, lb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    la.record(stream)
+    for _ in range(10):
+        dbuf.copy_(hbuf, non_blocking=True)
+    lb.record(stream)
+    torch.cuda.synchronize(dev)
+    link_gbs = 10 * hbuf.numel() / (la.elapsed_time(lb) * 1e-3) / 1e9
+    del dbuf
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    torch.cuda.synchronize(dev)
+    for i in range(args.steps):
+        cold_prep(i)
+        starts[i].record(stream)
+        step()
+        ends[i].record(stream)
+    torch.cuda.synchronize(dev)
+    total_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends))
+    cold_stats = [t.stats() for t in tabs]
+    # Warm: persistent caches, no flush, back to back.
+    step()
+    wa, wb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    wa.record(stream)
+    for i in range(args.steps):
+        step()
+    wb.record(stream)
+    torch.cuda.synchronize(dev)
+    warm_ms = wa.elapsed_time(wb) / args.steps
+    warm_stats = [t.stats() for t in tabs]
+    # Per-kernel durations of table 0 (cold, one table at a time).
+    t0 = tabs[0]
+    t0.trace_enable(True)
+    t0.trace_read()
+    for i in range(min(args.steps, 20)):
+        cold_prep(i)
+        sc, pr, wt, mk = outs[0]
+        t0.lookup_inject(q, K, hidden[:L], w.keep_ratio, scene_out=sc, prim_out=pr, weight_out=wt, mask_out=mk)
+    torch.cuda.synchronize(dev)
+    recs = t0.trace_read(max_records=400)
+    t0.trace_enable(False)
+    clocks = sampler.stop()
+    for t in tabs:
+        assert t.device_status() == 0, "a device-side wait timed out"
+    per_kernel = {}
+    for name, ms in recs:
+        per_kernel.setdefault(name, []).append(ms)
+    kernels_ms = {k: statistics.mean(v) for k, v in per_kernel.items()}
+    ms_per_step = total_ms / args.steps
+    stage_ms = kernels_ms.get("stage")
+    stage_gbs = stats[0]["staged_bytes"] / (stage_ms * 1e-3) / 1e9 if stage_ms else None
+    peaks, peak_kind = load_peaks()
+    result = {
+        "metric": METRIC, "value": N / (ms_per_step * 1e-3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": w.dtype, "data": "synthetic (seeded Gaussian mixture, random tables)",
+        "config": {"workload": w.name, "tokens": N, "tables": T, "layers_per_table": L, "d_key": w.d_key,
+                   "scenes": w.n_scenes, "prims": w.n_prims, "d_value": w.d_value, "top_k": K,
+                   "keep_ratio": w.keep_ratio, "residency": "pinned host, HBM slot cache per table",
+                   "l2": "cold: slot caches emptied and L2 flushed before every step, outside the events",
+                   "launch": f"one lookme_lookup_inject per table, tables alternating over {PIPE_STREAMS} streams"},
+        "roofline": {"bound": "host link", "staged_key_bytes_per_step": staged,
+                     "achieved": staged / (ms_per_step * 1e-3) / 1e9, "peak": link_gbs, "unit": "GB/s",
+                     "frac": staged / (ms_per_step * 1e-3) / 1e9 / link_gbs,
+                     "peak_source": "pinned host -> HBM copy-engine transfer of 256 MiB, measured in this run",
+                     "stage_kernel_gbs": stage_gbs},
+        "routed_scenes_per_table": routed, "selected_tokens_per_table": n_sel,
+        "cold_staged_bytes": sum(s["staged_bytes"] for s in cold_stats),
+        "warm": {"ms_per_step": warm_ms, "value": N / (warm_ms * 1e-3),
+                 "staged_bytes": sum(s["staged_bytes"] for s in warm_stats),
+                 "hits": sum(s["staged_hits"] for s in warm_stats)},
+        "link_gbs": link_gbs, "kernels_ms_table0": kernels_ms, "gpu_launches": launches_per_step * args.steps,
+        "clocks": clocks, "hbm_peak": float(peaks["hbm_gbs"]), "peak_kind": peak_kind,
+    }
+    for t in tabs:
+        t.close()
+    return result
+
+
 def oracle_step(o, data, idx, w):
     """The oracle's whole path on the tokens idx (route, level 2, selection over all priorities, injection)."""
     import numpy as np
@@ -605,7 +765,7 @@ def main():
 
         torch.cuda.set_device(local)
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    res = run_lookme(args, w, ws, rank, local)
+    res = run_multitable(args, w, ws, rank, local) if w.n_tables > 1 else run_lookme(args, w, ws, rank, local)
     if rank == 0:
         if ws == 1 and not args.no_cpu_baseline:
             res["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
