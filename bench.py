@@ -59,6 +59,9 @@ def parse():
     ap.add_argument("--impl", default="lookme", choices=["lookme", "reference"])
     ap.add_argument("--workload", default="single_image")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--replicas", type=int, default=0,
+                    help="table replicas the timed steps rotate through (0: as many as keep L2 cold; "
+                         "1: one table, L2 flushed before every step, e.g. for small profiler captures)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle baseline")
     return ap.parse_args()
 
@@ -81,8 +84,11 @@ def load_peaks():
 
 # The sources each profiled kernel is built from (the hash ties an ncu summary to them).
 KERNEL_SOURCES = {
-    "score": ["k_score_tc.cu", "score_tc.cuh", "topk.cuh", "sm100.cuh"],
-    "step": ["k_step.cu", "score_tc.cuh", "topk.cuh", "sm100.cuh"],
+    "score": ["k_score_tc.cu", "score_tc.cuh", "topk.cuh", "sm100.cuh", "common.cuh"],
+    "route": ["k_route.cu", "sm100.cuh", "common.cuh"],
+    "inject": ["k_inject.cu", "select.cuh", "common.cuh"],
+    "stage": ["k_stage.cu", "common.cuh"],
+    "step": ["k_step.cu", "score_tc.cuh", "topk.cuh", "sm100.cuh", "common.cuh"],
 }
 
 
@@ -231,7 +237,9 @@ def run_lookme(args, w, ws, rank, local):
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
 
-    R = plan_replicas(w)
+    R = plan_replicas(w) if args.replicas <= 0 else args.replicas
+    if R > 1 and R % PIPE_STREAMS:
+        raise SystemExit(f"--replicas must be 1 or a multiple of {PIPE_STREAMS}")
     tabs = [lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=w.dtype, device=local,
                          max_tokens=w.n_tokens) for _ in range(R)]
     cent = W.centroids(w, 0, dev)
