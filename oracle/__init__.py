@@ -206,3 +206,170 @@ def bf16_bits_to_f32(bits):
     """Widen bf16 bit patterns (uint16) to float32 values (exact)."""
     b = np.ascontiguousarray(bits, dtype=np.uint16).astype(np.uint32) << 16
     return b.view(np.float32)
+
+
+# ---------------------------------------------------------------------------
+# Second part (lookme_oracle_ext.c): the paper-exact level 2 with the MLP
+# ranker, the SKA gate, the text pathway, the dense ends and the multi-scale
+# router.  Same rules: test infrastructure only.
+_SRC_EXT = os.path.join(_HERE, "lookme_oracle_ext.c")
+_LIB_EXT = os.path.join(_HERE, "liblookme_oracle_ext.so")
+_lib_ext = None
+
+_SIGS_EXT = {
+    "lkx_linear": [_I64, _I64, _I64, _P, _P, _P, _P],
+    "lkx_ranker_relevance": [_I64, _I64, _I64, _I64, _I64, _P, _P, _P, _P, _P, _P, _P, _I32, _P],
+    "lkx_ranked_level2": [_I64, _I64, _I64, _I32, _P, _P, _P, _P, _P, _P, _P, _P, _P],
+    "lkx_ranked_weights_for": [_I64, _I64, _I64, _I32, _P, _P, _P, _P, _P, _P, _P],
+    "lkx_ska_gate": [_I64, _I64, _P, _P, _P, _P],
+    "lkx_combine": [_I64, _I64, _I64, _I32, _P, _P, _P, _P, _P, _P],
+    "lkx_text_inject": [_I64, _I64, _I64, _P, _P, _P, _I32, _P, _P],
+    "lkx_swiglu": [_I64, _I64, _I64, _I64, _P, _P, _P, _P, _I32, _P],
+    "lkx_propagate": [_I64, _I64, _P, _P, _P],
+    "lkx_scale_router": [_I64, _I64, _I64, _I32, _P, _P, _P, _P, _P],
+}
+
+
+def build_ext(force: bool = False, src: str = _SRC_EXT, out: str = _LIB_EXT) -> str:
+    """Compile the second part of the C oracle (gcc -O2 -fopenmp)."""
+    return build(force, src, out)
+
+
+def load_ext(path: str | None = None):
+    """Build (if needed) and load the second part; a path loads that file instead."""
+    global _lib_ext
+    if path is not None:
+        lib = ctypes.CDLL(path)
+        for name, argtypes in _SIGS_EXT.items():
+            fn = getattr(lib, name)
+            fn.argtypes = argtypes
+            fn.restype = None
+        return lib
+    with _lock:
+        if _lib_ext is None:
+            _lib_ext = load_ext(build_ext())
+    return _lib_ext
+
+
+def _i32(a):
+    return np.ascontiguousarray(a, dtype=np.int32)
+
+
+class PaperOracle:
+    """numpy front end to lookme_oracle_ext.c.  ``lib`` may be a mutated build (tests)."""
+
+    def __init__(self, lib=None):
+        self.lib = lib if lib is not None else load_ext()
+
+    def linear(self, x, W, b=None):
+        """x W^T + b with W [dout][din] (float64 result)."""
+        x, W = _f32(x), _f32(W)
+        n, din = x.shape
+        dout = W.shape[0]
+        assert W.shape[1] == din
+        y = np.empty((n, dout), np.float64)
+        self.lib.lkx_linear(n, din, dout, _ptr(x), _ptr(W), _ptr(None if b is None else _f32(b)), _ptr(y))
+        return y
+
+    def ranker_relevance(self, v, scene, cent, W1, b1, W2, b2, round_hidden=True):
+        """r = W2 silu(W1 [v ; e_img[scene]] + b1) + b2 (Level-2, first equation) [N][P]."""
+        v, cent, W1, b1, W2, b2 = (_f32(a) for a in (v, cent, W1, b1, W2, b2))
+        N, de = v.shape
+        S = cent.shape[0]
+        dm, P = W1.shape[0], W2.shape[0]
+        assert W1.shape[1] == 2 * de and W2.shape[1] == dm
+        r = np.empty((N, P), np.float64)
+        self.lib.lkx_ranker_relevance(N, S, de, dm, P, _ptr(v), _ptr(_i32(scene)), _ptr(cent), _ptr(W1), _ptr(b1),
+                                      _ptr(W2), _ptr(b2), 1 if round_hidden else 0, _ptr(r))
+        return r
+
+    def ranked_level2(self, v, scene, key_blocks, r, top_t, block_of_scene=None, n_scene=None):
+        """Top-T by r, weights softmax(cos + tanh r).  Returns dict(prim, weight, gap_T, gap_adj)."""
+        v = _f32(v)
+        N, de = v.shape
+        kb = np.asarray(key_blocks)
+        P = kb.shape[1]
+        kb, bos = _blocks(kb, block_of_scene, n_scene if n_scene is not None else kb.shape[0])
+        r = np.ascontiguousarray(r, dtype=np.float64)
+        if not 1 <= top_t <= min(P, 64):
+            raise ValueError("top_t out of range")
+        prim = np.empty((N, top_t), np.int32)
+        weight = np.empty((N, top_t), np.float64)
+        gap_T, gap_adj = np.empty(N, np.float64), np.empty(N, np.float64)
+        self.lib.lkx_ranked_level2(N, P, de, top_t, _ptr(v), _ptr(_i32(scene)), _ptr(kb), _ptr(bos), _ptr(r),
+                                   _ptr(prim), _ptr(weight), _ptr(gap_T), _ptr(gap_adj))
+        return dict(prim=prim, weight=weight, gap_T=gap_T, gap_adj=gap_adj)
+
+    def ranked_weights_for(self, v, scene, prim, key_blocks, r, block_of_scene=None, n_scene=None):
+        """The cos + tanh softmax of a given primitive set (conditional oracle)."""
+        v = _f32(v)
+        N, de = v.shape
+        kb = np.asarray(key_blocks)
+        P = kb.shape[1]
+        kb, bos = _blocks(kb, block_of_scene, n_scene if n_scene is not None else kb.shape[0])
+        prim = _i32(prim)
+        r = np.ascontiguousarray(r, dtype=np.float64)
+        w = np.empty(prim.shape, np.float64)
+        self.lib.lkx_ranked_weights_for(N, P, de, prim.shape[1], _ptr(v), _ptr(_i32(scene)), _ptr(prim), _ptr(kb),
+                                        _ptr(bos), _ptr(r), _ptr(w))
+        return w
+
+    def ska_gate(self, delta, wg):
+        """Hard SKA gate: returns (gate u8 [N], logit float64 [N])."""
+        delta, wg = _f32(delta), _f32(wg)
+        N, dh = delta.shape
+        gate, logit = np.empty(N, np.uint8), np.empty(N, np.float64)
+        self.lib.lkx_ska_gate(N, dh, _ptr(delta), _ptr(wg), _ptr(gate), _ptr(logit))
+        return gate, logit
+
+    def combine(self, scene, prim, weight, value_blocks, block_of_scene=None, n_scene=None):
+        """R_t = sum_j w_tj V[scene_t, prim_tj] (float64 [N][dv])."""
+        vb = np.asarray(value_blocks)
+        P, dv = vb.shape[1], vb.shape[2]
+        vb, bos = _blocks(vb, block_of_scene, n_scene if n_scene is not None else vb.shape[0])
+        prim = _i32(prim)
+        N, T = prim.shape
+        R = np.empty((N, dv), np.float64)
+        self.lib.lkx_combine(N, P, dv, T, _ptr(_i32(scene)), _ptr(prim),
+                             _ptr(np.ascontiguousarray(weight, dtype=np.float64)), _ptr(vb), _ptr(bos), _ptr(R))
+        return R
+
+    def text_inject(self, E, ids, gate, hidden):
+        """h + E[ids] on gated text positions of every layer (float64 [L][N][d])."""
+        E, hidden = _f32(E), _f32(hidden)
+        if hidden.ndim == 2:
+            hidden = hidden[None]
+        L, N, d = hidden.shape
+        out = np.empty((L, N, d), np.float64)
+        g = None if gate is None else np.ascontiguousarray(gate, dtype=np.uint8)
+        self.lib.lkx_text_inject(N, E.shape[0], d, _ptr(E), _ptr(_i32(ids)), _ptr(g), L, _ptr(hidden), _ptr(out))
+        return out
+
+    def swiglu(self, x, Wa, Wb, Wo, round_mid=True):
+        """(silu(x Wa^T) * (x Wb^T)) Wo^T (float64)."""
+        x, Wa, Wb, Wo = (_f32(a) for a in (x, Wa, Wb, Wo))
+        n, de = x.shape
+        dff, dh = Wa.shape[0], Wo.shape[0]
+        y = np.empty((n, dh), np.float64)
+        self.lib.lkx_swiglu(n, de, dff, dh, _ptr(x), _ptr(Wa), _ptr(Wb), _ptr(Wo), 1 if round_mid else 0, _ptr(y))
+        return y
+
+    def propagate(self, R, Wp):
+        """R W_p + R (W_p [de][de], paper orientation)."""
+        R, Wp = _f32(R), _f32(Wp)
+        n, de = R.shape
+        out = np.empty((n, de), np.float64)
+        self.lib.lkx_propagate(n, de, _ptr(R), _ptr(Wp), _ptr(out))
+        return out
+
+    def scale_router(self, H, Whe, Rs):
+        """Token-wise softmax router over M scales.  Returns (out [N][de], att [N][M])."""
+        H, Whe, Rs = _f32(H), _f32(Whe), _f32(Rs)
+        N, dh = H.shape
+        de = Whe.shape[1]
+        M = Rs.shape[0]
+        if not 1 <= M <= 64:
+            raise ValueError("1 <= M <= 64")
+        out, att = np.empty((N, de), np.float64), np.empty((N, M), np.float64)
+        self.lib.lkx_scale_router(N, dh, de, M, _ptr(H), _ptr(Whe), _ptr(Rs), _ptr(out), _ptr(att))
+        return out, att
