@@ -257,6 +257,131 @@ const char* lookme_kernel_name(int32_t kernel);
 lookme_status lookme_route_scenes_static(lookme_table* table, const void* queries, int64_t n_tokens,
                                          int32_t* scene_out, lookme_stream stream);
 
+/* ------------------------------------------------------------------------
+ * Paper-exact level 2 (Sec. "Level-2: scene-primitive retrieval").
+ *
+ * Install the scene-shared two-layer MLP ranker of a bf16 table:
+ *   r_j = W2 silu(W1 [v_e ; e_img[j]] + b1) + b2     (first equation)
+ *   W1  [d_hidden][2 d_key] bf16 (columns [0, d_key) multiply the query,
+ *       [d_key, 2 d_key) the scene's centroid), b1 [d_hidden] fp32,
+ *   W2  [n_prims][d_hidden] bf16, b2 [n_prims] fp32; host or device memory,
+ *       copied (the sources may be reused once the stream reaches the call).
+ * The activation is SiLU (the paper does not name it).  The per-scene term
+ * W1[:, d_key:] e_img[j] + b1 is computed by the next lookme_lookup_ranked
+ * and again after any lookme_load_scenes.  Synchronous when it replaces an
+ * earlier ranker.  Errors: INVALID_ARG (d_hidden not a multiple of 8 in
+ * [8, 4096], NULL weights), UNSUPPORTED (fp32 table), OOM, CUDA. */
+lookme_status lookme_set_ranker(lookme_table* table, int64_t d_hidden, const void* W1, const float* b1,
+                                const void* W2, const float* b2, lookme_stream stream);
+
+/* Level 1 as lookme_lookup, then the paper's level 2: the ranker's relevance
+ * r_t over the scene's n_prims primitives (two bf16 GEMMs on the tensor
+ * cores, the hidden activations rounded to bf16), the top_t primitives of
+ * largest r (ties: lower index; output in descending r), and the weights
+ *   w = softmax over the selected of cos(q_t, K[scene_t, p]) + tanh(r_t[p])
+ * (second equation; K is the table's keys, read only for the selected rows).
+ *   queries [n_tokens][d_key] bf16, scene_out [n_tokens], prim_out and
+ *   weight_out [n_tokens][top_t] (device).
+ * The table keeps ||q_t|| for lookme_inject's default priority.
+ * Errors: INVALID_ARG, STATE (no ranker, scenes not loaded, or scratch must
+ * grow under stream capture), OOM, CUDA. */
+lookme_status lookme_lookup_ranked(lookme_table* table, const void* queries, int64_t n_tokens, int32_t top_t,
+                                   int32_t* scene_out, int32_t* prim_out, float* weight_out, lookme_stream stream);
+
+/* SKA gate at inference (Sec. "Intra-Layer Sparse Activation", first
+ * equation): g_t = 1 exactly when sigmoid(Delta_t . w_g) > 0.5, i.e.
+ * Delta_t . w_g > 0 (the Gumbel-Sigmoid without noise).
+ *   delta [n_tokens][d_hidden], w_g [d_hidden] (dtype: LOOKME_BF16 or
+ *   LOOKME_FP32, d_hidden a multiple of 8 or 4), gate_out [n_tokens] u8,
+ *   logit_out [n_tokens] fp32 or NULL; device memory, current device.
+ * Errors: INVALID_ARG, CUDA. */
+lookme_status lookme_ska_gate(const void* delta, const void* w_g, int64_t n_tokens, int64_t d_hidden, int32_t dtype,
+                              uint8_t* gate_out, float* logit_out, lookme_stream stream);
+
+/* Sparse injection on a given gate (Sec. "Intra-Layer Sparse Activation",
+ * second equation, f the identity): for every t with gate[t] != 0,
+ *   h_l[t] += sum_j weight[t][j] V[scene[t], prim[t][j]]   for each layer l,
+ * accumulated in fp32 and rounded once; other rows are not touched.
+ *   scene [n_tokens], prim/weight [n_tokens][top_k], gate [n_tokens] u8,
+ *   hidden: host array of n_layers device pointers [n_tokens][d_value].
+ * Errors: INVALID_ARG, CUDA. */
+lookme_status lookme_inject_gated(lookme_table* table, const int32_t* scene, const int32_t* prim, const float* weight,
+                                  int64_t n_tokens, int32_t top_k, const uint8_t* gate, void* const* hidden,
+                                  int32_t n_layers, lookme_stream stream);
+
+/* Retrieved embeddings of listed tokens, the input of the fusion f:
+ *   R_out[i] = sum_j weight[t][j] V[scene[t], prim[t][j]],  t = rows[i]
+ * in fp32, written as bf16 [n_rows][d_value] (bf16 tables); scene, prim and
+ * weight are a lookup's outputs for n_tokens tokens, and a row id outside
+ * [0, n_tokens) yields a row of zeros.
+ * Errors: INVALID_ARG, UNSUPPORTED (fp32 table), CUDA. */
+lookme_status lookme_combine(lookme_table* table, const int32_t* scene, const int32_t* prim, const float* weight,
+                             int64_t n_tokens, int32_t top_k, const int32_t* rows, int64_t n_rows, void* R_out,
+                             lookme_stream stream);
+
+/* Text pathway (Sec. "Text", and the text-only PLE equation of Sec.
+ * "Method"): R_text = E_text[u], injected on the gated text positions:
+ *   h_l[t] += E[ids[t]] for every layer l, when (gate is NULL or gate[t])
+ *   and 0 <= ids[t] < vocab; positions whose id is outside the vocabulary
+ *   (image positions, say -1) are left untouched.
+ *   E [vocab][d] and hidden [n_tokens][d] in dtype (bf16 or fp32), ids
+ *   [n_tokens] int32, gate [n_tokens] u8 or NULL; device memory.
+ * Errors: INVALID_ARG, CUDA. */
+lookme_status lookme_text_inject(const void* E, int64_t vocab, int64_t d, int32_t dtype, const int32_t* ids,
+                                 const uint8_t* gate, int64_t n_tokens, void* const* hidden, int32_t n_layers,
+                                 lookme_stream stream);
+
+/* Projection into the embedding space (Sec. "Level-1": v_e = v W_{v->e}):
+ *   out[N][d_out] (bf16) = x[N][d_in] W^T + bias,
+ * with W [d_out][d_in] bf16 (the transpose of the paper's d_v x d_e matrix:
+ * a linear layer's weight) and bias [d_out] fp32 or NULL; tensor cores,
+ * fp32 accumulation.  d_in and d_out multiples of 8.  Errors: INVALID_ARG, CUDA. */
+lookme_status lookme_project(const void* x, const void* W, const float* bias, int64_t n_tokens, int64_t d_in,
+                             int64_t d_out, void* out, lookme_stream stream);
+
+/* Token-wise softmax router over the multi-scale results (Sec. "Multi-scale
+ * image retrieval"):
+ *   q_t = H_t W_he^T,  a_tm = softmax_m(q_t . R^m_t / sqrt(d_embed)),
+ *   out_t = sum_m a_tm R^m_t.
+ *   H [n_tokens][d_hidden] bf16; W_he [d_embed][d_hidden] bf16 (the
+ *   transpose of the paper's W_{h->e}); R_scales: host array of n_scales
+ *   (<= 16) device pointers [n_tokens][d_embed] bf16; workspace
+ *   [n_tokens][d_embed] fp32 (caller-owned, receives q); out
+ *   [n_tokens][d_embed] bf16; att_out [n_tokens][n_scales] fp32 or NULL.
+ * Errors: INVALID_ARG, CUDA. */
+lookme_status lookme_scale_router(const void* H, const void* W_he, const void* const* R_scales, int32_t n_scales,
+                                  int64_t n_tokens, int64_t d_hidden, int64_t d_embed, float* workspace, void* out,
+                                  float* att_out, lookme_stream stream);
+
+/* Fusion f and inter-layer propagation (Sec. "Intra-Layer Sparse
+ * Activation", second equation; Sec. "Inter-Layer Sparse Activation"): a
+ * stack of n_stages layers sharing one retrieval.  Stage 0 is the LookME
+ * layer, stage k >= 1 the k-th layer after it:
+ *   R^(0) = R,  R^(k) = R^(k-1) W_p^k + R^(k-1),
+ *   h_k[rows[i]] += f^k(R^(k)_i),  f^k(x) = (silu(x W_a^T) * (x W_b^T)) W_o^T,
+ * on tensor cores with fp32 accumulation; R^(k) and the SwiGLU product are
+ * rounded to bf16 between the GEMMs.  The object owns its weights and
+ * scratch (rows up to max_rows).  bf16 only; d_embed and d_hidden multiples
+ * of 8, d_ff a multiple of 32. */
+typedef struct lookme_fusion lookme_fusion;
+lookme_status lookme_fusion_create(int32_t n_stages, int64_t d_embed, int64_t d_ff, int64_t d_hidden, int32_t device,
+                                   int64_t max_rows, lookme_fusion** out);
+/* Weights of one stage, copied (host or device memory): W_a and W_b
+ * [d_ff][d_embed], W_o [d_hidden][d_ff], W_p [d_embed][d_embed] given as a
+ * linear layer's weight, i.e. the transpose of the paper's W_p (NULL for
+ * stage 0).  Errors: INVALID_ARG, CUDA. */
+lookme_status lookme_fusion_load(lookme_fusion* fusion, int32_t stage, const void* W_a, const void* W_b,
+                                 const void* W_o, const void* W_p, lookme_stream stream);
+/* R [n_rows][d_embed] bf16 (e.g. from lookme_combine), rows [n_rows] the
+ * token of each row (distinct), hidden: host array of n_stages device
+ * pointers [n_tokens][d_hidden] bf16, updated in place on the listed rows.
+ * Errors: INVALID_ARG, STATE (a stage without weights), CUDA. */
+lookme_status lookme_fusion_apply(lookme_fusion* fusion, const void* R, const int32_t* rows, int64_t n_rows,
+                                  void* const* hidden, lookme_stream stream);
+/* The fusion's device status word (bounded-wait timeouts), synchronously. */
+lookme_status lookme_fusion_status(lookme_fusion* fusion, uint32_t* status, lookme_stream stream);
+lookme_status lookme_fusion_destroy(lookme_fusion* fusion);
+
 const char* lookme_status_string(lookme_status status);
 const char* lookme_last_error(void);
 

@@ -19,7 +19,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "liblookme.so")
-SOURCES = ["lookme_api.cu", "k_route.cu", "k_bucket.cu", "k_score.cu", "k_score_tc.cu", "k_inject.cu", "k_stage.cu", "k_step.cu"]
+SOURCES = ["lookme_api.cu", "k_route.cu", "k_bucket.cu", "k_score.cu", "k_score_tc.cu", "k_inject.cu", "k_stage.cu", "k_step.cu", "k_gemm_tc.cu", "k_dense_misc.cu", "lookme_dense.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr", f"-I{INCLUDE}", f"-I{CSRC}"]

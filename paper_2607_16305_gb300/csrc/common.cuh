@@ -32,6 +32,14 @@ enum KernelId : int32_t {
     KID_BUCKET_SCATTER = 15,  // K2 for large calls: token ids into their items
     KID_STEP = 16,            // K1 + K2 + K3 (+ gate and K4): the fused step on tcgen05
     KID_STAGE_ASSIGN = 17,    // K6a: slot cache look-up and the copy list
+    KID_GEMM = 18,            // dense bf16 GEMM (ranker MLP, projection, fusion, propagation, router)
+    KID_DECODE = 19,          // argmax key -> scene, key reset (paper-exact level 2)
+    KID_RANKED_SELECT = 20,   // top-T by relevance, cos + tanh softmax
+    KID_SKA_GATE = 21,        // hard SKA gate
+    KID_INJECT_GATED = 22,    // injection on a given gate
+    KID_TEXT_INJECT = 23,     // text pathway gather + injection
+    KID_COMBINE = 24,         // retrieved embeddings of listed tokens
+    KID_ROUTER = 25,          // multi-scale softmax router
     KID_COUNT
 };
 
@@ -291,6 +299,69 @@ cudaError_t launch_stage_assign(const LaunchCtx& c, const StageArgs& sa, const i
                                 const int32_t* counters, WorkItem* work, uint32_t* status);
 cudaError_t launch_stage(const LaunchCtx& c, const void* keys_host_mapped, void* slots, int64_t block_bytes,
                          const StageArgs& sa);
+
+// ----------------------------------------------- dense bf16 GEMM on tcgen05
+// D[M][Nn] = A[M][K] B[Nn][K]^T (bf16 operands, fp32 accumulation in TMEM),
+// with one of these epilogues:
+enum GemmEpi : int {
+    EPI_F32 = 0,          // out f32 = D + colbias
+    EPI_BF16 = 1,         // out bf16 = act(D + colbias + rowbias[rowsel[m]])
+    EPI_SWIGLU = 2,       // out bf16 [M][Nn/2] = silu(gate) * up, B rows interleaved per 32 features
+    EPI_RESID = 3,        // out bf16 = D + colbias + resid (resid may be out itself)
+    EPI_SCATTER_ADD = 4,  // out[rowidx[m]] (bf16) += D + colbias
+};
+struct GemmArgs {
+    int64_t M, Nn, K;
+    int mode, act;            // act: 0 none, 1 silu (EPI_BF16)
+    const float* colbias;     // [Nn] or null
+    const float* rowbias;     // [..][ld_rowbias], row rowsel[m] (EPI_BF16) or null
+    const int32_t* rowsel;
+    int64_t ld_rowbias;
+    void* out;
+    int64_t ld_out;           // elements
+    const void* resid;        // bf16 [M][ld_resid] (EPI_RESID)
+    int64_t ld_resid;
+    const int32_t* rowidx;    // destination rows (EPI_SCATTER_ADD)
+    uint32_t* status;         // bounded waits report here (bit STATUS_IN_GEMM)
+};
+constexpr uint32_t STATUS_IN_GEMM = 32u;
+// Tile width chosen for (M, Nn) on num_sms SMs: 64, 128 or 256 columns.
+int gemm_tile_n(int64_t M, int64_t Nn, int num_sms);
+// tmap_a: [M][K] bf16, box 64 x 128 rows; tmap_b: [Nn][K] bf16, box 64 x BN rows
+// (BN = gemm_tile_n), both with the 128-byte swizzle.
+cudaError_t launch_gemm_tc(const LaunchCtx& c, const void* tmap_a, const void* tmap_b, int bn, const GemmArgs& g);
+cudaError_t configure_gemm_kernels();
+
+// ------------------------------------------------ SIMT kernels around GEMMs
+// scene_out[t] = the routed scene of argmax key best[t]; best[t] reset to 0.
+cudaError_t launch_decode_reset(const LaunchCtx& c, unsigned long long* best, int64_t N, int64_t S,
+                                int32_t* scene_out);
+// Keys of a bf16 table as stored: tiled (the level-2 kernel's layout) or row-major.
+struct KeyView {
+    const uint8_t* keys;
+    int64_t block_bytes;  // bytes per scene
+    int P, dk;
+    int tiled, ntile, nkb;
+};
+// Paper-exact level 2 from the relevance r [N][P] (fp32): top-T per token,
+// weights softmax(cos(q, K[scene, p]) + tanh r[p]); one warp per token.
+cudaError_t launch_ranked_select(const LaunchCtx& c, const float* r, int64_t ld_r, int64_t N, int T, const __nv_bfloat16* q,
+                                 const KeyView& kv, const int32_t* scene, int32_t* prim_out, float* weight_out);
+// g_t = [Delta_t . w_g > 0]; logit_out optional.
+cudaError_t launch_ska_gate(const LaunchCtx& c, int dtype, const void* delta, const void* wg, int64_t N, int64_t dh,
+                            uint8_t* gate, float* logit_out);
+// h_l[t] += sum_j w_tj V[scene_t, prim_tj] for every t with gate[t].
+cudaError_t launch_inject_gated(const LaunchCtx& c, const InjectArgs& a, const uint8_t* gate);
+// h_l[t] += E[ids[t]] for gated t with 0 <= ids[t] < V.
+cudaError_t launch_text_inject(const LaunchCtx& c, int dtype, const void* E, int64_t V, int64_t d,
+                               const int32_t* ids, const uint8_t* gate, int64_t N, void* const* hidden, int n_layers);
+// R_out[i] (bf16) = sum_j w_tj V[scene_t, prim_tj], t = rows[i].
+cudaError_t launch_combine(const LaunchCtx& c, const InjectArgs& a, const int32_t* rows, int64_t n,
+                           __nv_bfloat16* R_out);
+// out_t = sum_m softmax_m(q_t . R^m_t / sqrt(de)) R^m_t; q fp32 [N][de], R^m bf16 [N][de].
+constexpr int kRouterMaxScales = 16;
+cudaError_t launch_scale_router(const LaunchCtx& c, const float* q, const __nv_bfloat16* const* Rs, int M, int64_t N,
+                                int64_t de, __nv_bfloat16* out, float* att_out);
 
 // ------------------------------------------------------------- fused step
 // Routing, bucketing, level 2, the injection gate and the injection in one

@@ -27,6 +27,9 @@ EXPORTS = [
     "lookme_reserve", "lookme_stage_invalidate", "lookme_last_lookup_stats", "lookme_device_status", "lookme_launch_count",
     "lookme_trace_enable", "lookme_trace_read", "lookme_kernel_name", "lookme_status_string",
     "lookme_last_error", "lookme_route_scenes_static", "lookme_lookup_inject",
+    "lookme_set_ranker", "lookme_lookup_ranked", "lookme_ska_gate", "lookme_inject_gated", "lookme_combine",
+    "lookme_text_inject", "lookme_project", "lookme_scale_router", "lookme_fusion_create", "lookme_fusion_load",
+    "lookme_fusion_apply", "lookme_fusion_status", "lookme_fusion_destroy",
 ]
 
 
@@ -85,6 +88,19 @@ def load(path: str = LIB_PATH):
         "lookme_last_error": ([], ctypes.c_char_p),
         "lookme_route_scenes_static": ([P, P, I64, P, P], I32),
         "lookme_lookup_inject": ([P, P, I64, I32, P, P, I32, D, P, I32, P, P, P, P, P], I32),
+        "lookme_set_ranker": ([P, I64, P, P, P, P, P], I32),
+        "lookme_lookup_ranked": ([P, P, I64, I32, P, P, P, P], I32),
+        "lookme_ska_gate": ([P, P, I64, I64, I32, P, P, P], I32),
+        "lookme_inject_gated": ([P, P, P, P, I64, I32, P, P, I32, P], I32),
+        "lookme_combine": ([P, P, P, P, I64, I32, P, I64, P, P], I32),
+        "lookme_text_inject": ([P, I64, I64, I32, P, P, I64, P, I32, P], I32),
+        "lookme_project": ([P, P, P, I64, I64, I64, P, P], I32),
+        "lookme_scale_router": ([P, P, P, I32, I64, I64, I64, P, P, P, P], I32),
+        "lookme_fusion_create": ([I32, I64, I64, I64, I32, I64, ctypes.POINTER(P)], I32),
+        "lookme_fusion_load": ([P, I32, P, P, P, P, P], I32),
+        "lookme_fusion_apply": ([P, P, P, I64, P, P], I32),
+        "lookme_fusion_status": ([P, ctypes.POINTER(ctypes.c_uint32), P], I32),
+        "lookme_fusion_destroy": ([P], I32),
     }
     for name, (argtypes, restype) in sig.items():
         fn = getattr(lib, name)
@@ -262,3 +278,146 @@ class Table:
         n = ctypes.c_int32()
         _check(self.lib.lookme_trace_read(self.handle, buf, max_records, ctypes.byref(n)))
         return [(self.lib.lookme_kernel_name(buf[i].kernel).decode(), buf[i].ms) for i in range(n.value)]
+
+
+# ------------------------------------------------------------------------------
+# The pieces around the two-level lookup (Sec. "Level-2", "Text", "Sparse
+# Injection", "Multi-scale image retrieval"): thin marshalling, as above.
+def _ptrs(ts):
+    return (ctypes.c_void_p * len(ts))(*[t.data_ptr() for t in ts])
+
+
+def _set_ranker(self, W1, b1, W2, b2, stream=None):
+    """Install the ranker MLP: W1 [d_m, 2 d_key] bf16, b1 [d_m] fp32, W2 [n_prims, d_m] bf16, b2 [n_prims] fp32."""
+    for name, t, dt in (("W1", W1, torch.bfloat16), ("b1", b1, torch.float32), ("W2", W2, torch.bfloat16),
+                        ("b2", b2, torch.float32)):
+        self._tensor(t, name, dt, device=False)
+    _check(self.lib.lookme_set_ranker(self.handle, W1.shape[0], _ptr(W1), _ptr(b1), _ptr(W2), _ptr(b2),
+                                      _stream(stream, self.device)))
+
+
+def _lookup_ranked(self, queries, top_t, scene_out=None, prim_out=None, weight_out=None, stream=None):
+    """Level 1, then the paper's level 2 (MLP relevance, top-T, cos + tanh softmax)."""
+    self._tensor(queries, "queries", self.torch_dtype)
+    N, dev = queries.shape[0], self.device
+    scene_out = torch.empty(N, dtype=torch.int32, device=dev) if scene_out is None else scene_out
+    prim_out = torch.empty(N, top_t, dtype=torch.int32, device=dev) if prim_out is None else prim_out
+    weight_out = torch.empty(N, top_t, dtype=torch.float32, device=dev) if weight_out is None else weight_out
+    _check(self.lib.lookme_lookup_ranked(self.handle, _ptr(queries), N, top_t, _ptr(scene_out), _ptr(prim_out),
+                                         _ptr(weight_out), _stream(stream, dev)))
+    return scene_out, prim_out, weight_out
+
+
+def _inject_gated(self, scene, prim, weight, gate, hidden, stream=None):
+    """h_l[t] += sum_j w V rows for every gated t (in place)."""
+    hidden = list(hidden) if isinstance(hidden, (list, tuple)) else [hidden]
+    for i, h in enumerate(hidden):
+        self._tensor(h, f"hidden[{i}]", self.torch_dtype)
+    N, k = prim.shape
+    _check(self.lib.lookme_inject_gated(self.handle, _ptr(scene), _ptr(prim), _ptr(weight), N, k, _ptr(gate),
+                                        _ptrs(hidden), len(hidden), _stream(stream, self.device)))
+
+
+def _combine(self, scene, prim, weight, rows, out=None, stream=None):
+    """Retrieved embeddings of the listed tokens, bf16 [len(rows), d_value]."""
+    n, k = rows.shape[0], prim.shape[1]
+    out = torch.empty(n, self.shape[3], dtype=torch.bfloat16, device=self.device) if out is None else out
+    _check(self.lib.lookme_combine(self.handle, _ptr(scene), _ptr(prim), _ptr(weight), scene.shape[0], k, _ptr(rows),
+                                   n, _ptr(out), _stream(stream, self.device)))
+    return out
+
+
+Table.set_ranker = _set_ranker
+Table.lookup_ranked = _lookup_ranked
+Table.inject_gated = _inject_gated
+Table.combine = _combine
+
+
+def _code(dtype):
+    return BF16 if dtype == torch.bfloat16 else FP32
+
+
+def ska_gate(delta, w_g, gate_out=None, logit_out=None, stream=None):
+    """Hard SKA gate g = [delta . w_g > 0]; returns (gate u8, logit fp32 or None)."""
+    lib = load()
+    N, dh = delta.shape
+    gate_out = torch.empty(N, dtype=torch.uint8, device=delta.device) if gate_out is None else gate_out
+    _check(lib.lookme_ska_gate(_ptr(delta), _ptr(w_g), N, dh, _code(delta.dtype), _ptr(gate_out), _ptr(logit_out),
+                               _stream(stream, delta.device)))
+    return gate_out, logit_out
+
+
+def text_inject(E, ids, hidden, gate=None, stream=None):
+    """h_l[t] += E[ids[t]] on gated text positions (ids outside [0, V) are skipped); in place."""
+    lib = load()
+    hidden = list(hidden) if isinstance(hidden, (list, tuple)) else [hidden]
+    V, d = E.shape
+    _check(lib.lookme_text_inject(_ptr(E), V, d, _code(E.dtype), _ptr(ids), _ptr(gate), ids.shape[0], _ptrs(hidden),
+                                  len(hidden), _stream(stream, E.device)))
+
+
+def project(x, W, bias=None, out=None, stream=None):
+    """x W^T + bias in bf16 on the tensor cores (W [d_out, d_in])."""
+    lib = load()
+    N, d_in = x.shape
+    d_out = W.shape[0]
+    out = torch.empty(N, d_out, dtype=torch.bfloat16, device=x.device) if out is None else out
+    _check(lib.lookme_project(_ptr(x), _ptr(W), _ptr(bias), N, d_in, d_out, _ptr(out), _stream(stream, x.device)))
+    return out
+
+
+def scale_router(H, W_he, scales, out=None, att_out=None, workspace=None, stream=None):
+    """Softmax router over the scales' results (W_he [d_e, d_h]); returns (out bf16 [N, d_e], att or None)."""
+    lib = load()
+    N, dh = H.shape
+    de = W_he.shape[0]
+    workspace = torch.empty(N, de, dtype=torch.float32, device=H.device) if workspace is None else workspace
+    out = torch.empty(N, de, dtype=torch.bfloat16, device=H.device) if out is None else out
+    _check(lib.lookme_scale_router(_ptr(H), _ptr(W_he), _ptrs(scales), len(scales), N, dh, de, _ptr(workspace),
+                                   _ptr(out), _ptr(att_out), _stream(stream, H.device)))
+    return out, att_out
+
+
+class Fusion:
+    """SwiGLU fusion f and the R W_p + R propagation over n_stages layers (bf16)."""
+
+    def __init__(self, n_stages, d_embed, d_ff, d_hidden, device=0, max_rows=4096):
+        self.lib = load()
+        self.device = torch.device("cuda", device) if isinstance(device, int) else torch.device(device)
+        h = ctypes.c_void_p()
+        _check(self.lib.lookme_fusion_create(n_stages, d_embed, d_ff, d_hidden, self.device.index or 0, max_rows,
+                                             ctypes.byref(h)))
+        self.handle = h
+        self.n_stages = n_stages
+
+    def load_stage(self, stage, W_a, W_b, W_o, W_p=None, stream=None):
+        """W_a, W_b [d_ff, d_e]; W_o [d_h, d_ff]; W_p [d_e, d_e] as a linear weight (paper's W_p transposed)."""
+        _check(self.lib.lookme_fusion_load(self.handle, stage, _ptr(W_a), _ptr(W_b), _ptr(W_o), _ptr(W_p),
+                                           _stream(stream, self.device)))
+
+    def apply(self, R, rows, hidden, stream=None):
+        """h_k[rows] += f^k(R^(k)) for every stage k (in place)."""
+        _check(self.lib.lookme_fusion_apply(self.handle, _ptr(R), _ptr(rows), rows.shape[0], _ptrs(hidden),
+                                            _stream(stream, self.device)))
+
+    def status(self, stream=None):
+        v = ctypes.c_uint32()
+        _check(self.lib.lookme_fusion_status(self.handle, ctypes.byref(v), _stream(stream, self.device)))
+        return v.value
+
+    def close(self):
+        if getattr(self, "handle", None):
+            self.lib.lookme_fusion_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:  # noqa: BLE001 - interpreter shutdown
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()

@@ -1,0 +1,286 @@
+"""The paper-exact pieces around the lookup on the GPU, against the oracle's
+second part (lookme_oracle_ext.c), through the C ABI.
+
+Tolerances, from the arithmetic:
+  * GEMM outputs rounded to bf16: one bf16 rounding of an fp32 accumulation,
+    so within one bf16 ulp (2^-8 relative) of the exactly rounded value.
+  * Ranker relevance: the hidden activations are rounded to bf16 on both
+    sides, but an fp32 and an fp64 pre-activation can straddle a rounding
+    midpoint and round one ulp apart; that moves r by at most
+    sum_m |W2[p,m]| ulp(h_m).  Primitive sets must match except where the
+    oracle's own gap r_(T) - r_(T+1) is below RANK_TIE (counted); weights
+    (a softmax of cos + tanh r) within W_TOL of the oracle's weights of the
+    GPU's primitive set.
+  * Gate: exact except where |logit| < 1e-3 (fp32 vs fp64 dot product).
+  * Hidden rows: 2e-2 (bf16) / 1e-5 (fp32), the lookup's bar; untouched rows
+    bit-identical.
+"""
+from __future__ import annotations
+
+import numpy as np
+import pytest
+import torch
+
+import gpu_harness as H
+from paper_2607_16305_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+DEV = torch.device("cuda", 0) if torch.cuda.is_available() else None
+RANK_TIE = 1e-2
+W_TOL = 2e-3
+
+
+@pytest.fixture(scope="module")
+def paper_oracle():
+    import oracle as oracle_pkg
+
+    return oracle_pkg.PaperOracle()
+
+
+def _g(seed):
+    g = torch.Generator(device=DEV)
+    g.manual_seed(seed)
+    return g
+
+
+def _rand(shape, seed, scale=1.0, dtype=torch.bfloat16):
+    return (scale * torch.randn(*shape, generator=_g(seed), device=DEV)).to(dtype).contiguous()
+
+
+def _bf16_ulp(x):
+    x = np.abs(np.asarray(x, np.float64))
+    e = np.floor(np.log2(np.maximum(x, 2.0 ** -126)))
+    return 2.0 ** (e - 7)
+
+
+# ---------------------------------------------------------------- projection
+@pytest.mark.parametrize("N,d_in,d_out", [(1, 8, 8), (300, 136, 200), (1024, 256, 512), (129, 520, 64),
+                                          (2000, 64, 1032)])
+def test_project_gemm(lookme_lib, paper_oracle, N, d_in, d_out):
+    """x W^T + b through the tcgen05 GEMM: every tile width, ragged M, N and K."""
+    from paper_2607_16305_gb300 import lookme
+
+    x = _rand((N, d_in), 1)
+    Wt = _rand((d_out, d_in), 2, 0.1)
+    b = _rand((d_out,), 3, 0.5, torch.float32)
+    out = lookme.project(x, Wt, b)
+    torch.cuda.synchronize()
+    ref = paper_oracle.linear(H.f32(x), H.f32(Wt), H.f32(b))
+    got = H.f32(out)
+    err = np.abs(got - ref)
+    assert (err <= _bf16_ulp(ref) + 1e-6).all(), f"max error {err.max()}"
+
+
+# ------------------------------------------------------- paper-exact level 2
+def _ranker_weights(de, dm, P, seed=7):
+    W1 = _rand((dm, 2 * de), seed, 1.0 / np.sqrt(2 * de))
+    b1 = _rand((dm,), seed + 1, 0.1, torch.float32)
+    W2 = _rand((P, dm), seed + 2, 2.0 / np.sqrt(dm))
+    b2 = _rand((P,), seed + 3, 0.1, torch.float32)
+    return W1, b1, W2, b2
+
+
+RANKED_CASES = [
+    ("r1", dict(n_tokens=300, n_scenes=40, n_prims=64, d_key=128, d_value=64, top_k=8, keep_ratio=0.25), 64),
+    ("r2", dict(n_tokens=1, n_scenes=1, n_prims=8, d_key=16, d_value=8, top_k=8, keep_ratio=1.0), 8),
+    ("r3", dict(n_tokens=517, n_scenes=70, n_prims=200, d_key=64, d_value=32, top_k=16, keep_ratio=0.25), 104),
+    ("r4", dict(n_tokens=256, n_scenes=16, n_prims=256, d_key=256, d_value=64, top_k=8, keep_ratio=0.5), 256),
+]
+
+
+@pytest.mark.parametrize("name,kw,dm", RANKED_CASES, ids=[c[0] for c in RANKED_CASES])
+def test_lookup_ranked(oracle, lookme_lib, paper_oracle, name, kw, dm):
+    from paper_2607_16305_gb300 import lookme
+
+    w = W.small(name, **kw)
+    with lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype="bf16", device=0) as t:
+        cent = H.load_table(t, w, 0, DEV)
+        W1, b1, W2, b2 = _ranker_weights(w.d_key, dm, w.n_prims)
+        t.set_ranker(W1, b1, W2, b2)
+        q = W.queries(w, DEV)
+        scene, prim, weight = t.lookup_ranked(q, w.top_k)
+        torch.cuda.synchronize()
+        assert t.device_status() == 0
+        # Twice more: the per-scene term is cached; results are identical.
+        s2, p2, w2 = t.lookup_ranked(q, w.top_k)
+        torch.cuda.synchronize()
+        assert torch.equal(scene, s2) and torch.equal(prim, p2) and torch.equal(weight, w2)
+    qs, cent_np = H.f32(q), H.f32(cent)
+    gscene, gprim, gw = scene.cpu().numpy(), prim.cpu().numpy(), weight.cpu().numpy()
+    r = oracle.route(qs, cent_np)
+    bad = (gscene != r["scene"]) & (r["gap1"] >= 1e-3)
+    assert not bad.any(), f"{int(bad.sum())} scene mismatches"
+    kb, kbos = H.scene_blocks(w, np.arange(w.n_scenes), 0, DEV, None, cent, "keys")
+    rel = paper_oracle.ranker_relevance(qs, gscene, cent_np, H.f32(W1), H.f32(b1), H.f32(W2), H.f32(b2), True)
+    ref = paper_oracle.ranked_level2(qs, gscene, kb, rel, w.top_k)
+    assert ((gprim >= 0) & (gprim < w.n_prims)).all()
+    assert all(len(set(row)) == w.top_k for row in gprim.tolist())
+    same = (np.sort(gprim, 1) == np.sort(ref["prim"], 1)).all(1)
+    flagged = ref["gap_T"] < RANK_TIE
+    assert (same | flagged).all(), f"{int((~same & ~flagged).sum())} primitive-set mismatches outside the band"
+    ordered = same & (ref["gap_adj"] >= RANK_TIE)
+    assert (gprim[ordered] == ref["prim"][ordered]).all(), "primitive order differs"
+    wref = paper_oracle.ranked_weights_for(qs, gscene, gprim, kb, rel)
+    assert np.abs(gw - wref).max() <= W_TOL, f"weights max error {np.abs(gw - wref).max()}"
+    assert np.abs(gw.sum(1) - 1).max() <= 1e-5
+    print(f"{name}: set ties {int((~same).sum())} flagged {int(flagged.sum())} w err {np.abs(gw - wref).max():.2e}")
+
+
+def test_lookup_ranked_errors(lookme_lib):
+    from paper_2607_16305_gb300 import lookme
+
+    w = W.small("rerr", n_tokens=16, n_scenes=4, n_prims=16, d_key=32, d_value=16, top_k=4, keep_ratio=0.25)
+    with lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype="bf16", device=0) as t:
+        H.load_table(t, w, 0, DEV)
+        q = W.queries(w, DEV)
+        with pytest.raises(lookme.LookmeError):
+            t.lookup_ranked(q, 4)  # no ranker yet
+        W1, b1, W2, b2 = _ranker_weights(w.d_key, 12, w.n_prims)
+        with pytest.raises(lookme.LookmeError):
+            t.set_ranker(W1, b1, W2, b2)  # d_hidden not a multiple of 8
+        W1, b1, W2, b2 = _ranker_weights(w.d_key, 16, w.n_prims)
+        t.set_ranker(W1, b1, W2, b2)
+        with pytest.raises(lookme.LookmeError):
+            t.lookup_ranked(q, 17)  # top_t > n_prims
+        t.lookup_ranked(q, 4)
+        torch.cuda.synchronize()
+    with lookme.Table(4, 16, 32, 16, dtype="fp32", device=0) as t:
+        with pytest.raises(lookme.LookmeError):
+            t.set_ranker(W1, b1, W2, b2)  # fp32 table
+
+
+# --------------------------------------------------------- gate and injection
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+def test_ska_gate_and_gated_injection(oracle, lookme_lib, paper_oracle, dtype):
+    from paper_2607_16305_gb300 import lookme
+
+    w = W.small(f"gate_{dtype}", n_tokens=400, n_scenes=30, n_prims=32, d_key=64, d_value=128, top_k=4,
+                keep_ratio=0.25, dtype=dtype)
+    tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    delta = _rand((w.n_tokens, w.d_value), 11, 1.0, tdt)
+    wg = _rand((w.d_value,), 12, 1.0 / np.sqrt(w.d_value), tdt)
+    logit = torch.empty(w.n_tokens, dtype=torch.float32, device=DEV)
+    gate, _ = lookme.ska_gate(delta, wg, logit_out=logit)
+    torch.cuda.synchronize()
+    og, ol = paper_oracle.ska_gate(H.f32(delta), H.f32(wg))
+    gg = gate.cpu().numpy()
+    assert np.abs(logit.cpu().numpy() - ol).max() <= 1e-4
+    diff = gg != og
+    assert (np.abs(ol[diff]) < 1e-3).all(), "gate differs away from 0"
+    assert 0 < gg.sum() < w.n_tokens
+    with lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=dtype, device=0) as t:
+        cent = H.load_table(t, w, 0, DEV)
+        q = W.queries(w, DEV)
+        scene, prim, weight = t.lookup(q, w.top_k)
+        hs = [W.hidden(w, l, DEV) for l in range(2)]
+        h0 = [h.clone() for h in hs]
+        t.inject_gated(scene, prim, weight, gate, hs)
+        torch.cuda.synchronize()
+    keep = gate.bool()
+    for l in range(2):
+        assert torch.equal(hs[l][~keep], h0[l][~keep])
+    rows = np.nonzero(gg)[0]
+    gscene = scene.cpu().numpy()[rows]
+    vb, vbos = H.scene_blocks(w, gscene, 0, DEV, None, cent, "values")
+    ref = oracle.inject(gscene, prim.cpu().numpy()[rows], weight.cpu().numpy()[rows].astype(np.float64),
+                        np.ones(rows.size, np.uint8), vb, np.stack([H.f32(h)[rows] for h in h0]), vbos, w.n_scenes)
+    got = np.stack([H.f32(h)[rows] for h in hs])
+    assert np.abs(got - ref).max() <= H.hidden_tol(dtype)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+def test_text_inject(lookme_lib, paper_oracle, dtype):
+    from paper_2607_16305_gb300 import lookme
+
+    tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    V, d, N = 1000, 256, 700
+    E = _rand((V, d), 21, 0.05, tdt)
+    ids = torch.randint(-5, V + 5, (N,), generator=_g(22), device=DEV, dtype=torch.int32)
+    gate = (torch.rand(N, generator=_g(23), device=DEV) < 0.6).to(torch.uint8)
+    hs = [_rand((N, d), 24 + l, 1.0, tdt) for l in range(3)]
+    h0 = [h.clone() for h in hs]
+    lookme.text_inject(E, ids, hs, gate=gate)
+    torch.cuda.synchronize()
+    ref = paper_oracle.text_inject(H.f32(E), ids.cpu().numpy(), gate.cpu().numpy(), np.stack([H.f32(h) for h in h0]))
+    if dtype == "bf16":
+        import oracle as oracle_pkg
+
+        want = oracle_pkg.bf16_bits_to_f32(oracle_pkg.Oracle().round_bf16(ref))
+        assert np.array_equal(np.stack([H.f32(h) for h in hs]), want), "bf16 text injection not exactly rounded"
+    else:
+        assert np.abs(np.stack([H.f32(h) for h in hs]) - ref).max() <= 1e-5
+    # No gate: every text position.
+    hs = [h.clone() for h in h0]
+    lookme.text_inject(E, ids, hs)
+    torch.cuda.synchronize()
+    ref = paper_oracle.text_inject(H.f32(E), ids.cpu().numpy(), None, np.stack([H.f32(h) for h in h0]))
+    assert np.abs(np.stack([H.f32(h) for h in hs]) - ref).max() <= H.hidden_tol(dtype)
+
+
+# ----------------------------------------------------- fusion and propagation
+def test_combine_and_fusion(oracle, lookme_lib, paper_oracle):
+    import oracle as oracle_pkg
+    from paper_2607_16305_gb300 import lookme
+
+    w = W.small("fuse", n_tokens=600, n_scenes=24, n_prims=32, d_key=64, d_value=256, top_k=8, keep_ratio=0.25)
+    de, dff, dh, n_st = w.d_value, 512, 384, 3
+    ob = oracle_pkg.Oracle()
+
+    def rb(x):
+        return oracle_pkg.bf16_bits_to_f32(ob.round_bf16(x))
+
+    with lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype="bf16", device=0) as t:
+        cent = H.load_table(t, w, 0, DEV)
+        q = W.queries(w, DEV)
+        scene, prim, weight = t.lookup(q, w.top_k)
+        rows = torch.nonzero(torch.rand(w.n_tokens, generator=_g(31), device=DEV) < 0.3).flatten().to(torch.int32)
+        R = t.combine(scene, prim, weight, rows)
+        torch.cuda.synchronize()
+    rws = rows.cpu().numpy()
+    gscene = scene.cpu().numpy()[rws]
+    vb, vbos = H.scene_blocks(w, gscene, 0, DEV, None, cent, "values")
+    Rref = paper_oracle.combine(gscene, prim.cpu().numpy()[rws], weight.cpu().numpy()[rws].astype(np.float64), vb,
+                                vbos, w.n_scenes)
+    assert np.abs(H.f32(R) - Rref).max() <= np.max(_bf16_ulp(Rref)) * 0.5 + 1e-7
+    Wa = [_rand((dff, de), 40 + k, 1 / np.sqrt(de)) for k in range(n_st)]
+    Wb = [_rand((dff, de), 50 + k, 1 / np.sqrt(de)) for k in range(n_st)]
+    Wo = [_rand((dh, dff), 60 + k, 1 / np.sqrt(dff)) for k in range(n_st)]
+    Wp = [None] + [_rand((de, de), 70 + k, 0.5 / np.sqrt(de)) for k in range(1, n_st)]  # linear weights
+    hs = [_rand((w.n_tokens, dh), 80 + k) for k in range(n_st)]
+    h0 = [h.clone() for h in hs]
+    with lookme.Fusion(n_st, de, dff, dh, device=0, max_rows=1024) as f:
+        for k in range(n_st):
+            f.load_stage(k, Wa[k], Wb[k], Wo[k], Wp[k])
+        f.apply(R, rows, hs)
+        torch.cuda.synchronize()
+        assert f.status() == 0
+    keep = torch.zeros(w.n_tokens, dtype=torch.bool, device=DEV)
+    keep[rows.long()] = True
+    Rk = H.f32(R)
+    for k in range(n_st):
+        assert torch.equal(hs[k][~keep], h0[k][~keep]), f"stage {k}: an unlisted row changed"
+        if k > 0:
+            # The kernel rounds R^(k) to bf16; the oracle's propagation takes the paper's W_p.
+            Rk = rb(paper_oracle.propagate(Rk, H.f32(Wp[k]).T.copy()))
+        y = paper_oracle.swiglu(Rk, H.f32(Wa[k]), H.f32(Wb[k]), H.f32(Wo[k]), round_mid=True)
+        ref = H.f32(h0[k])[rws].astype(np.float64) + y
+        err = np.abs(H.f32(hs[k])[rws] - ref).max()
+        assert err <= 2e-2, f"stage {k}: hidden max error {err}"
+
+
+# --------------------------------------------------------------- the router
+def test_scale_router(lookme_lib, paper_oracle):
+    from paper_2607_16305_gb300 import lookme
+
+    N, dh, de, M = 700, 384, 256, 3
+    Hs = _rand((N, dh), 91)
+    Whe = _rand((de, dh), 92, 1 / np.sqrt(dh))
+    Rs = [_rand((N, de), 93 + m, 0.5) for m in range(M)]
+    att = torch.empty(N, M, dtype=torch.float32, device=DEV)
+    out, _ = lookme.scale_router(Hs, Whe, Rs, att_out=att)
+    torch.cuda.synchronize()
+    oout, oatt = paper_oracle.scale_router(H.f32(Hs), H.f32(Whe).T.copy(), np.stack([H.f32(r) for r in Rs]))
+    assert np.abs(att.cpu().numpy() - oatt).max() <= 1e-4
+    err = np.abs(H.f32(out) - oout)
+    assert (err <= _bf16_ulp(oout) + 1e-4).all(), f"router output max error {err.max()}"
