@@ -59,6 +59,9 @@ def parse():
     ap.add_argument("--impl", default="lookme", choices=["lookme", "reference"])
     ap.add_argument("--workload", default="single_image")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--path", default="keys", choices=("keys",) + PATHS,
+                    help="keys: the two-level lookup + injection (the default step); the others time one of the "
+                         "paper-exact pieces on the single-image sizes")
     ap.add_argument("--replicas", type=int, default=0,
                     help="table replicas the timed steps rotate through (0: as many as keep L2 cold; "
                          "1: one table, L2 flushed before every step, e.g. for small profiler captures)")
@@ -661,6 +664,196 @@ def run_multitable(args, w, ws, rank, local):
     return result
 
 
+# ------------------------------------------------------------------------------
+# Bench lines of the paper-exact pieces (--path): one call at a time, L2
+# flushed before each, events around it, on the single-image sizes (the
+# paper's own d_e = 512 for the embedding-space pieces).
+PATHS = ("ranked", "fusion", "router", "project", "text")
+
+
+def _time_calls(fn, steps, warmup, flush, stream, sampler=None):
+    import torch
+
+    for i in range(warmup):
+        flush(i)
+        fn()
+    torch.cuda.synchronize()
+    st = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    en = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    for i in range(steps):
+        flush(i)
+        st[i].record(stream)
+        fn()
+        en[i].record(stream)
+    torch.cuda.synchronize()
+    return statistics.mean(a.elapsed_time(b) for a, b in zip(st, en))
+
+
+def run_path(args, w):
+    """One of PATHS on the single-image sizes; returns the JSON line."""
+    import torch
+
+    from __graft_entry__ import build
+    from paper_2607_16305_gb300 import lookme
+    from paper_2607_16305_gb300 import workloads as W
+
+    build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(0)
+    stream = torch.cuda.current_stream(dev)
+    flush_buf = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
+    sink = torch.zeros((), dtype=torch.int64, device=dev)
+
+    def flush(i):
+        flush_buf.fill_(i & 0xFF)
+        sink.copy_(flush_buf.sum(dtype=torch.int64))
+
+    def rnd(shape, seed, scale=1.0, dtype=torch.bfloat16):
+        g = torch.Generator(device=dev)
+        g.manual_seed(seed)
+        return (scale * torch.randn(*shape, generator=g, device=dev)).to(dtype).contiguous()
+
+    peaks, peak_kind = load_peaks()
+    hbm, tf = float(peaks["hbm_gbs"]), float(peaks["bf16_tflops"])
+    N, K = w.n_tokens, w.top_k
+    launches = None
+    kernels = {}
+    sampler = ClockSampler(0)
+    sampler.start()
+    if args.path == "ranked":
+        dm = 256
+        t = lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=w.dtype, device=0, max_tokens=N)
+        cent = W.centroids(w, 0, dev)
+        for c in range(w.n_chunks):
+            k, v = W.table_chunk(w, 0, c, dev, None, cent)
+            t.load_scenes(c * w.scenes_per_chunk, k, v, centroids=cent[c * w.scenes_per_chunk:][:k.shape[0]])
+            del k, v
+        t.set_ranker(rnd((dm, 2 * w.d_key), 1, 1 / math.sqrt(2 * w.d_key)), rnd((dm,), 2, 0.1, torch.float32),
+                     rnd((w.n_prims, dm), 3, 2 / math.sqrt(dm)), rnd((w.n_prims,), 4, 0.1, torch.float32))
+        q = W.queries(w, dev)
+        delta = rnd((N, w.d_value), 5)
+        wg = rnd((w.d_value,), 6, 1 / math.sqrt(w.d_value))
+        hidden = [W.hidden(w, 0, dev)]
+        sc = torch.empty(N, dtype=torch.int32, device=dev)
+        pr = torch.empty(N, K, dtype=torch.int32, device=dev)
+        wt = torch.empty(N, K, dtype=torch.float32, device=dev)
+        gate = torch.empty(N, dtype=torch.uint8, device=dev)
+
+        def fn():
+            lookme.ska_gate(delta, wg, gate_out=gate)
+            t.lookup_ranked(q, K, scene_out=sc, prim_out=pr, weight_out=wt)
+            t.inject_gated(sc, pr, wt, gate, hidden)
+
+        fn()
+        torch.cuda.synchronize()
+        n_sel = int(gate.sum().item())
+        c0 = t.launch_count()
+        fn()
+        torch.cuda.synchronize()
+        launches = t.launch_count() - c0 + 1  # + the gate kernel (table-less)
+        ms = _time_calls(fn, args.steps, args.warmup, flush, stream)
+        t.trace_enable(True)
+        t.trace_read()
+        _time_calls(fn, min(args.steps, 50), 1, flush, stream)
+        for name, v in t.trace_read(max_records=2000):
+            kernels.setdefault(name, []).append(v)
+        t.trace_enable(False)
+        e = w.elem_bytes
+        nbytes = (N * w.d_key * e + w.n_scenes * w.d_key * e + N * K * w.d_key * e + N * w.d_value * e
+                  + dm * (2 * w.d_key + w.n_prims) * e + n_sel * K * w.d_value * e + 2 * n_sel * w.d_value * e)
+        flops = 2 * N * w.n_scenes * w.d_key + 2 * N * (w.d_key * dm + dm * w.n_prims)
+        what = f"SKA gate + level 1 + MLP-ranked level 2 (d_m {dm}, top-{K}) + gated injection"
+        t.close()
+    elif args.path == "fusion":
+        de, dff, dh, n_st, n = 512, 2048, w.d_value, 4, N // 4
+        f = lookme.Fusion(n_st, de, dff, dh, device=0, max_rows=n)
+        for k in range(n_st):
+            f.load_stage(k, rnd((dff, de), 10 + k, 1 / math.sqrt(de)), rnd((dff, de), 20 + k, 1 / math.sqrt(de)),
+                         rnd((dh, dff), 30 + k, 1 / math.sqrt(dff)),
+                         rnd((de, de), 40 + k, 0.5 / math.sqrt(de)) if k else None)
+        R = rnd((n, de), 50, 0.05)
+        rows = torch.arange(0, N, 4, dtype=torch.int32, device=dev)
+        hidden = [rnd((N, dh), 60 + k) for k in range(n_st)]
+
+        def fn():
+            f.apply(R, rows, hidden)
+
+        ms = _time_calls(fn, args.steps, args.warmup, flush, stream)
+        assert f.status() == 0
+        launches = 3 * n_st - 1
+        flops = n_st * (2 * n * de * 2 * dff + 2 * n * dff * dh) + (n_st - 1) * 2 * n * de * de
+        nbytes = 2 * (n_st * (2 * dff * de + dh * dff) + (n_st - 1) * de * de) + n * de * 2 + n_st * 2 * n * dh * 2
+        what = f"SwiGLU fusion d_e {de} -> d_ff {dff} -> d_h {dh} on {n} gated tokens, {n_st} layers with R W_p + R"
+        f.close()
+    elif args.path == "router":
+        de, dh, M = 512, w.d_value, 3
+        Hs = rnd((N, dh), 70)
+        Whe = rnd((de, dh), 71, 1 / math.sqrt(dh))
+        Rs = [rnd((N, de), 72 + m, 0.5) for m in range(M)]
+        out = torch.empty(N, de, dtype=torch.bfloat16, device=dev)
+        ws = torch.empty(N, de, dtype=torch.float32, device=dev)
+
+        def fn():
+            lookme.scale_router(Hs, Whe, Rs, out=out, workspace=ws)
+
+        ms = _time_calls(fn, args.steps, args.warmup, flush, stream)
+        launches = 2
+        flops = 2 * N * dh * de
+        nbytes = N * dh * 2 + de * dh * 2 + M * N * de * 2 + N * de * 2 + 2 * N * de * 4
+        what = f"multi-scale softmax router over {M} scales (d_h {dh} -> d_e {de})"
+    elif args.path == "project":
+        dv, de = w.d_value, 512
+        x = rnd((N, dv), 80)
+        Wv = rnd((de, dv), 81, 1 / math.sqrt(dv))
+        out = torch.empty(N, de, dtype=torch.bfloat16, device=dev)
+
+        def fn():
+            lookme.project(x, Wv, out=out)
+
+        ms = _time_calls(fn, args.steps, args.warmup, flush, stream)
+        launches = 1
+        flops = 2 * N * dv * de
+        nbytes = N * dv * 2 + de * dv * 2 + N * de * 2
+        what = f"projection W_v->e ({dv} -> {de})"
+    else:  # text
+        V, d = 151936, w.d_value
+        E = rnd((V, d), 90, 0.02)
+        g = torch.Generator(device=dev)
+        g.manual_seed(91)
+        ids = torch.randint(0, V, (N,), generator=g, device=dev, dtype=torch.int32)
+        ids[::2] = -1  # image positions
+        gate = (torch.rand(N, generator=g, device=dev) < 0.5).to(torch.uint8)
+        hidden = [rnd((N, d), 92 + l) for l in range(4)]
+
+        def fn():
+            lookme.text_inject(E, ids, hidden, gate=gate)
+
+        ms = _time_calls(fn, args.steps, args.warmup, flush, stream)
+        n_on = int(((ids >= 0) & (gate > 0)).sum().item())
+        launches = 1
+        flops = 0
+        nbytes = N * 5 + n_on * d * 2 * (1 + 2 * len(hidden))
+        what = f"text ID lookup (vocab {V}, d {d}) injected into {len(hidden)} layers"
+    clocks = sampler.stop()
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    tfs = flops / (ms * 1e-3) / 1e12
+    t_bytes, t_flops = nbytes / hbm / 1e9, flops / tf / 1e12
+    bound = "hbm" if t_bytes >= t_flops else "tensor"
+    roof = {"bound": bound, "unit": "GB/s" if bound == "hbm" else "TFLOP/s",
+            "achieved": gbs if bound == "hbm" else tfs, "peak": hbm if bound == "hbm" else tf,
+            "algorithmic_bytes": nbytes, "algorithmic_flops": flops, "peak_source": peak_kind,
+            "roofline_us": max(t_bytes, t_flops) * 1e6}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    return {"metric": METRIC, "value": N / (ms * 1e-3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded Gaussian mixture, random weights)",
+            "config": {"workload": w.name, "path": args.path, "what": what, "tokens": N,
+                       "l2": f"flushed before every call ({FLUSH_BYTES >> 20} MiB written then read, outside the events)",
+                       "launch": "one call at a time, events around it"},
+            "roofline": roof, "kernels_ms": {k: statistics.mean(v) for k, v in kernels.items()},
+            "gpu_launches": launches * args.steps if launches else None, "clocks": clocks, "cpu_baseline": None}
+
+
 def oracle_step(o, data, idx, w):
     """The oracle's whole path on the tokens idx (route, level 2, selection over all priorities, injection)."""
     import numpy as np
@@ -766,6 +959,10 @@ def main():
     if args.impl == "reference":
         if rank == 0:
             print(json.dumps(run_reference(args, w)), flush=True)
+        return
+    if args.path != "keys":
+        if rank == 0:
+            print(json.dumps(run_path(args, w)), flush=True)
         return
     if ws > 1:
         import torch

@@ -70,7 +70,16 @@ __global__ void __launch_bounds__(kr::kWarps * 32) k_ranked_select(const float* 
     const int P = kv.P;
     const float* rt = r + t * ld_r;
     // Top-T by r, larger first, lower primitive on ties: T rounds of a warp
-    // argmax over the entries after the previous winner in that order.
+    // argmax over the entries after the previous winner in that order.  A
+    // lane's entries (p = lane + 32 i) are read once, up to 64 of them into
+    // registers (P <= 2,048); larger P re-reads the row from L1.
+    constexpr int kReg = 8;
+    float rl[kReg];
+#pragma unroll
+    for (int i = 0; i < kReg; ++i) {
+        const int p = lane + 32 * i;
+        rl[i] = p < P ? rt[p] : -INFINITY;
+    }
     int sel[LOOKME_MAX_TOP_K];
     float rv[LOOKME_MAX_TOP_K];
     float last_v = INFINITY;
@@ -78,7 +87,17 @@ __global__ void __launch_bounds__(kr::kWarps * 32) k_ranked_select(const float* 
     for (int j = 0; j < T; ++j) {
         float bv = -INFINITY;
         int bp = INT_MAX;
-        for (int p = lane; p < P; p += 32) {
+#pragma unroll
+        for (int i = 0; i < kReg; ++i) {
+            const int p = lane + 32 * i;
+            const float v = rl[i];
+            const bool after = v < last_v || (v == last_v && p > last_p);
+            if (p < P && after && (v > bv || (v == bv && p < bp))) {
+                bv = v;
+                bp = p;
+            }
+        }
+        for (int p = lane + 32 * kReg; p < P; p += 32) {
             const float v = rt[p];
             const bool after = v < last_v || (v == last_v && p > last_p);
             if (after && (v > bv || (v == bv && p < bp))) {
@@ -113,22 +132,40 @@ __global__ void __launch_bounds__(kr::kWarps * 32) k_ranked_select(const float* 
     nq = sqrtf(kr::warp_sum(nq));
     float sc[LOOKME_MAX_TOP_K];
     float smax = -INFINITY;
-    for (int j = 0; j < T; ++j) {
-        float dot = 0.f, nk = 0.f;
-        for (int u = 0; u * 32 + lane < nch && u < 4; ++u) {
-            float kf[8];
-            Vec16<__nv_bfloat16>::unpack(*kr::key_chunk(kv, s, sel[j], u * 32 + lane), kf);
+    // Eight key rows at a time: every lane issues its chunk loads of the
+    // eight rows before any arithmetic, then the warp reduces each row.
+    for (int j0 = 0; j0 < T; j0 += 8) {
+        float dot[8], nk[8];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                dot = fmaf(qv[8 * u + e], kf[e], dot);
-                nk = fmaf(kf[e], kf[e], nk);
+        for (int jj = 0; jj < 8; ++jj) dot[jj] = nk[jj] = 0.f;
+        for (int u = 0; u * 32 + lane < nch && u < 4; ++u) {
+            uint4 kc[8];
+#pragma unroll
+            for (int jj = 0; jj < 8; ++jj)
+                if (j0 + jj < T) kc[jj] = *kr::key_chunk(kv, s, sel[j0 + jj], u * 32 + lane);
+#pragma unroll
+            for (int jj = 0; jj < 8; ++jj) {
+                if (j0 + jj < T) {
+                    float kf[8];
+                    Vec16<__nv_bfloat16>::unpack(kc[jj], kf);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        dot[jj] = fmaf(qv[8 * u + e], kf[e], dot[jj]);
+                        nk[jj] = fmaf(kf[e], kf[e], nk[jj]);
+                    }
+                }
             }
         }
-        dot = kr::warp_sum(dot);
-        nk = sqrtf(kr::warp_sum(nk));
-        const float cosv = (nq > 0.f && nk > 0.f) ? dot / (nq * nk) : 0.f;
-        sc[j] = cosv + tanhf(rv[j]);
-        smax = fmaxf(smax, sc[j]);
+#pragma unroll
+        for (int jj = 0; jj < 8; ++jj) {
+            if (j0 + jj < T) {
+                const float d = kr::warp_sum(dot[jj]);
+                const float n = sqrtf(kr::warp_sum(nk[jj]));
+                const float cosv = (nq > 0.f && n > 0.f) ? d / (nq * n) : 0.f;
+                sc[j0 + jj] = cosv + tanhf(rv[j0 + jj]);
+                smax = fmaxf(smax, sc[j0 + jj]);
+            }
+        }
     }
     float den = 0.f;
     for (int j = 0; j < T; ++j) {
@@ -221,13 +258,28 @@ __global__ void __launch_bounds__(256) k_gated_rows(const __grid_constant__ Gate
         float acc[V];
 #pragma unroll
         for (int e = 0; e < V; ++e) acc[e] = 0.f;
-        for (int j = 0; j < (valid ? p.top_k : 0); ++j) {
-            const int64_t row = s * p.P + p.prim[t * p.top_k + j];
-            const float w = p.weight[t * p.top_k + j];
-            float f[V];
-            Vec16<T>::unpack(reinterpret_cast<const uint4*>(vals + row * p.dv)[cidx], f);
+        const int kk = valid ? p.top_k : 0;
+        for (int j0 = 0; j0 < kk; j0 += 8) {
+            // Eight rows' chunks in flight before any is used.
+            uint4 c8[8];
+            float w8[8];
 #pragma unroll
-            for (int e = 0; e < V; ++e) acc[e] = fmaf(w, f[e], acc[e]);
+            for (int jj = 0; jj < 8; ++jj) {
+                if (j0 + jj < kk) {
+                    const int64_t row = s * p.P + p.prim[t * p.top_k + j0 + jj];
+                    w8[jj] = p.weight[t * p.top_k + j0 + jj];
+                    c8[jj] = reinterpret_cast<const uint4*>(vals + row * p.dv)[cidx];
+                }
+            }
+#pragma unroll
+            for (int jj = 0; jj < 8; ++jj) {
+                if (j0 + jj < kk) {
+                    float f[V];
+                    Vec16<T>::unpack(c8[jj], f);
+#pragma unroll
+                    for (int e = 0; e < V; ++e) acc[e] = fmaf(w8[jj], f[e], acc[e]);
+                }
+            }
         }
         if (kCombine) {
             uint4 o;
