@@ -721,49 +721,85 @@ def run_path(args, w):
     sampler = ClockSampler(0)
     sampler.start()
     if args.path == "ranked":
-        dm = 256
-        t = lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=w.dtype, device=0, max_tokens=N)
+        dm, R = 256, 10  # 10 table replicas (11.3 GiB) for the two-stream measurement, as for the keys path
+        W1, b1 = rnd((dm, 2 * w.d_key), 1, 1 / math.sqrt(2 * w.d_key)), rnd((dm,), 2, 0.1, torch.float32)
+        W2, b2 = rnd((w.n_prims, dm), 3, 2 / math.sqrt(dm)), rnd((w.n_prims,), 4, 0.1, torch.float32)
+        tabs = [lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=w.dtype, device=0, max_tokens=N)
+                for _ in range(R)]
         cent = W.centroids(w, 0, dev)
         for c in range(w.n_chunks):
             k, v = W.table_chunk(w, 0, c, dev, None, cent)
-            t.load_scenes(c * w.scenes_per_chunk, k, v, centroids=cent[c * w.scenes_per_chunk:][:k.shape[0]])
+            for t in tabs:
+                t.load_scenes(c * w.scenes_per_chunk, k, v, centroids=cent[c * w.scenes_per_chunk:][:k.shape[0]])
             del k, v
-        t.set_ranker(rnd((dm, 2 * w.d_key), 1, 1 / math.sqrt(2 * w.d_key)), rnd((dm,), 2, 0.1, torch.float32),
-                     rnd((w.n_prims, dm), 3, 2 / math.sqrt(dm)), rnd((w.n_prims,), 4, 0.1, torch.float32))
-        q = W.queries(w, dev)
-        delta = rnd((N, w.d_value), 5)
+        for t in tabs:
+            t.set_ranker(W1, b1, W2, b2)
+        q0 = W.queries(w, dev)
+        delta0 = rnd((N, w.d_value), 5)
         wg = rnd((w.d_value,), 6, 1 / math.sqrt(w.d_value))
-        hidden = [W.hidden(w, 0, dev)]
-        sc = torch.empty(N, dtype=torch.int32, device=dev)
-        pr = torch.empty(N, K, dtype=torch.int32, device=dev)
-        wt = torch.empty(N, K, dtype=torch.float32, device=dev)
-        gate = torch.empty(N, dtype=torch.uint8, device=dev)
+        bufs = [dict(q=q0.clone(), delta=delta0.clone(), hidden=[W.hidden(w, 0, dev)],
+                     sc=torch.empty(N, dtype=torch.int32, device=dev), pr=torch.empty(N, K, dtype=torch.int32, device=dev),
+                     wt=torch.empty(N, K, dtype=torch.float32, device=dev),
+                     gate=torch.empty(N, dtype=torch.uint8, device=dev)) for _ in range(R)]
+
+        def fn_r(r):
+            b_ = bufs[r]
+            lookme.ska_gate(b_["delta"], wg, gate_out=b_["gate"])
+            tabs[r].lookup_ranked(b_["q"], K, scene_out=b_["sc"], prim_out=b_["pr"], weight_out=b_["wt"])
+            tabs[r].inject_gated(b_["sc"], b_["pr"], b_["wt"], b_["gate"], b_["hidden"])
 
         def fn():
-            lookme.ska_gate(delta, wg, gate_out=gate)
-            t.lookup_ranked(q, K, scene_out=sc, prim_out=pr, weight_out=wt)
-            t.inject_gated(sc, pr, wt, gate, hidden)
+            fn_r(0)
 
-        fn()
+        for r in range(R):
+            fn_r(r)
         torch.cuda.synchronize()
-        n_sel = int(gate.sum().item())
+        t = tabs[0]
+        n_sel = int(bufs[0]["gate"].sum().item())
         c0 = t.launch_count()
         fn()
         torch.cuda.synchronize()
         launches = t.launch_count() - c0 + 1  # + the gate kernel (table-less)
-        ms = _time_calls(fn, args.steps, args.warmup, flush, stream)
+        latency_ms = _time_calls(fn, args.steps, args.warmup, flush, stream)
+        # Two batches in flight over the replicas (graphs of 64 steps), as the keys path's value.
+        streams = [torch.cuda.Stream(dev) for _ in range(2)]
+        gph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gph):
+            cur = torch.cuda.current_stream(dev)
+            for s_ in streams:
+                s_.wait_stream(cur)
+            for i in range(64):
+                with torch.cuda.stream(streams[i % 2]):
+                    fn_r(i % R)
+            for s_ in streams:
+                cur.wait_stream(s_)
+        for _ in range(2):
+            gph.replay()
+        torch.cuda.synchronize()
+        reps = max(1, args.steps // 64)
+        ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ea.record(stream)
+        for _ in range(reps):
+            gph.replay()
+        eb.record(stream)
+        torch.cuda.synchronize()
+        ms = ea.elapsed_time(eb) / (reps * 64)
         t.trace_enable(True)
         t.trace_read()
         _time_calls(fn, min(args.steps, 50), 1, flush, stream)
         for name, v in t.trace_read(max_records=2000):
             kernels.setdefault(name, []).append(v)
         t.trace_enable(False)
+        for tt in tabs:
+            assert tt.device_status() == 0
         e = w.elem_bytes
         nbytes = (N * w.d_key * e + w.n_scenes * w.d_key * e + N * K * w.d_key * e + N * w.d_value * e
                   + dm * (2 * w.d_key + w.n_prims) * e + n_sel * K * w.d_value * e + 2 * n_sel * w.d_value * e)
         flops = 2 * N * w.n_scenes * w.d_key + 2 * N * (w.d_key * dm + dm * w.n_prims)
-        what = f"SKA gate + level 1 + MLP-ranked level 2 (d_m {dm}, top-{K}) + gated injection"
-        t.close()
+        what = (f"SKA gate + level 1 + MLP-ranked level 2 (d_m {dm}, top-{K}) + gated injection; value: two "
+                f"batches in flight over {R} table replicas, {reps * 64} steps; latency: one call at a time")
+        for tt in tabs:
+            tt.close()
     elif args.path == "fusion":
         de, dff, dh, n_st, n = 512, 2048, w.d_value, 4, N // 4
         f = lookme.Fusion(n_st, de, dff, dh, device=0, max_rows=n)
@@ -844,7 +880,8 @@ def run_path(args, w):
             "algorithmic_bytes": nbytes, "algorithmic_flops": flops, "peak_source": peak_kind,
             "roofline_us": max(t_bytes, t_flops) * 1e6}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    return {"metric": METRIC, "value": N / (ms * 1e-3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+    extra = {"latency_ms_per_call": latency_ms} if args.path == "ranked" else {}
+    return {**extra, "metric": METRIC, "value": N / (ms * 1e-3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded Gaussian mixture, random weights)",
             "config": {"workload": w.name, "path": args.path, "what": what, "tokens": N,
