@@ -284,3 +284,116 @@ def test_scale_router(lookme_lib, paper_oracle):
     assert np.abs(att.cpu().numpy() - oatt).max() <= 1e-4
     err = np.abs(H.f32(out) - oout)
     assert (err <= _bf16_ulp(oout) + 1e-4).all(), f"router output max error {err.max()}"
+
+
+# ------------------------------------------------------------ more edge cases
+def test_ranked_on_pinned_host_table_and_graph(oracle, lookme_lib, paper_oracle):
+    """The paper-form level 2 on a pinned-host table (key rows read over the
+    host link), its default-priority injection, and a CUDA-graph replay."""
+    from paper_2607_16305_gb300 import lookme
+
+    w = W.small("rhost", n_tokens=300, n_scenes=40, n_prims=64, d_key=128, d_value=64, top_k=8, keep_ratio=0.25,
+                residency="host")
+    with lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype="bf16", residency="host", device=0,
+                      max_tokens=w.n_tokens) as t:
+        cent = H.load_table(t, w, 0, DEV)
+        W1, b1, W2, b2 = _ranker_weights(w.d_key, 64, w.n_prims)
+        t.set_ranker(W1, b1, W2, b2)
+        q = W.queries(w, DEV)
+        scene, prim, weight = t.lookup_ranked(q, w.top_k)
+        hs = [W.hidden(w, 0, DEV)]
+        h0 = hs[0].clone()
+        mask = t.inject(scene, prim, weight, hs, w.keep_ratio)
+        torch.cuda.synchronize()
+        # Graph capture of the ranked lookup replays to the same outputs.
+        so = torch.empty_like(scene)
+        po = torch.empty_like(prim)
+        wo = torch.empty_like(weight)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            t.lookup_ranked(q, w.top_k, scene_out=so, prim_out=po, weight_out=wo)
+        g.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(so, scene) and torch.equal(po, prim) and torch.equal(wo, weight)
+        assert t.device_status() == 0
+    qs = H.f32(q)
+    gscene, gprim, gw = scene.cpu().numpy(), prim.cpu().numpy(), weight.cpu().numpy()
+    kb, kbos = H.scene_blocks(w, np.arange(w.n_scenes), 0, DEV, None, cent, "keys")
+    rel = paper_oracle.ranker_relevance(qs, gscene, H.f32(cent), H.f32(W1), H.f32(b1), H.f32(W2), H.f32(b2), True)
+    ref = paper_oracle.ranked_level2(qs, gscene, kb, rel, w.top_k)
+    same = (np.sort(gprim, 1) == np.sort(ref["prim"], 1)).all(1)
+    assert (same | (ref["gap_T"] < RANK_TIE)).all()
+    wref = paper_oracle.ranked_weights_for(qs, gscene, gprim, kb, rel)
+    assert np.abs(gw - wref).max() <= W_TOL
+    # Injection on the default priority (||q||) with the ranked weights.
+    gm = mask.cpu().numpy()
+    H.check_mask(oracle, oracle.query_norms(qs), gm, w.keep_ratio, [0, w.n_tokens])
+    rows = np.nonzero(gm)[0]
+    vb, vbos = H.scene_blocks(w, gscene[rows], 0, DEV, None, cent, "values")
+    hr = oracle.inject(gscene[rows], gprim[rows], wref[rows], np.ones(rows.size, np.uint8), vb,
+                       H.f32(h0)[rows][None], vbos, w.n_scenes)
+    assert np.abs(H.f32(hs[0])[rows] - hr[0]).max() <= H.hidden_tol("bf16")
+    keep = mask.bool()
+    assert torch.equal(hs[0][~keep], h0[~keep])
+
+
+def test_fusion_single_stage_and_limits(lookme_lib, paper_oracle):
+    from paper_2607_16305_gb300 import lookme
+
+    de, dff, dh = 64, 96, 40
+    with lookme.Fusion(1, de, dff, dh, device=0, max_rows=3) as f:
+        Wa, Wb, Wo = _rand((dff, de), 101, 0.2), _rand((dff, de), 102, 0.2), _rand((dh, dff), 103, 0.2)
+        with pytest.raises(lookme.LookmeError):
+            f.apply(_rand((1, de), 104), torch.zeros(1, dtype=torch.int32, device=DEV), [_rand((5, dh), 105)])
+        f.load_stage(0, Wa, Wb, Wo)
+        R = _rand((1, de), 106)
+        rows = torch.tensor([3], dtype=torch.int32, device=DEV)
+        h = _rand((5, dh), 107)
+        h0 = h.clone()
+        f.apply(R, rows, [h])
+        torch.cuda.synchronize()
+        y = paper_oracle.swiglu(H.f32(R), H.f32(Wa), H.f32(Wb), H.f32(Wo), True)
+        assert np.abs(H.f32(h)[3] - (H.f32(h0)[3] + y[0])).max() <= 2e-2
+        assert torch.equal(h[[0, 1, 2, 4]], h0[[0, 1, 2, 4]])
+        with pytest.raises(lookme.LookmeError):
+            f.apply(_rand((4, de), 108), torch.arange(4, dtype=torch.int32, device=DEV), [h])  # > max_rows
+        assert f.status() == 0
+    with pytest.raises(lookme.LookmeError):
+        lookme.Fusion(1, de, 100, dh, device=0)  # d_ff not a multiple of 32
+
+
+@pytest.mark.parametrize("M", [1, 16])
+def test_scale_router_extremes(lookme_lib, paper_oracle, M):
+    from paper_2607_16305_gb300 import lookme
+
+    N, dh, de = 257, 64, 128
+    Hs = _rand((N, dh), 110)
+    Whe = _rand((de, dh), 111, 1 / np.sqrt(dh))
+    Rs = [_rand((N, de), 112 + m, 0.5) for m in range(M)]
+    att = torch.empty(N, M, dtype=torch.float32, device=DEV)
+    out, _ = lookme.scale_router(Hs, Whe, Rs, att_out=att)
+    torch.cuda.synchronize()
+    oout, oatt = paper_oracle.scale_router(H.f32(Hs), H.f32(Whe).T.copy(), np.stack([H.f32(r) for r in Rs]))
+    assert np.abs(att.cpu().numpy() - oatt).max() <= 1e-4
+    assert (np.abs(H.f32(out) - oout) <= _bf16_ulp(oout) + 1e-4).all()
+    if M == 1:
+        assert torch.equal(out, Rs[0])
+
+
+def test_dense_entry_point_errors(lookme_lib):
+    from paper_2607_16305_gb300 import lookme
+
+    x = _rand((8, 12), 120)
+    with pytest.raises(lookme.LookmeError):
+        lookme.project(x, _rand((8, 12), 121))  # d_in not a multiple of 8
+    with pytest.raises(lookme.LookmeError):
+        lookme.scale_router(_rand((4, 16), 122), _rand((16, 16), 123), [_rand((4, 16), 124)] * 17)  # > 16 scales
+    delta = _rand((4, 10), 125, 1.0, torch.float32)
+    with pytest.raises(lookme.LookmeError):
+        lookme.ska_gate(delta, _rand((10,), 126, 1.0, torch.float32))  # fp32 d_hidden not a multiple of 4
+    E = _rand((10, 16), 127)
+    h = [_rand((3, 16), 128)]
+    h0 = h[0].clone()
+    lookme.text_inject(E, torch.tensor([-1, 10, 99], dtype=torch.int32, device=DEV), h)  # no text positions
+    torch.cuda.synchronize()
+    assert torch.equal(h[0], h0)
