@@ -9,12 +9,14 @@ keep 25%) unless --workload says otherwise.
 
   value      tokens/s over K device-timed steps, inputs resident in HBM.  When
              the table is small enough to hold several copies (single image:
-             10 replicas, 11.3 GiB), step i runs on replica i % R and the steps
-             alternate over two streams, so two batches are in flight (one
-             batch's routing and bucketing beside the other's level 2); the
-             steps are replayed as CUDA graphs of 64 steps between one pair of
-             events, and R - 1 other steps pass between two uses of a replica,
-             so its data is out of L2 (inputs larger than L2, no flush).
+             12 replicas, 13.6 GiB), step i runs on replica i % R and the steps
+             rotate over S streams (single image: 6), so S batches are in
+             flight (some batches' routing, bucketing and injection beside
+             another's level 2), with the routing and bucketing grids sized
+             for 24 SMs (lookme_set_small_grid); the steps are replayed as CUDA
+             graphs of 64 steps between one pair of events, and R - 1 other
+             steps pass between two uses of a replica, so its data is out of
+             L2 (inputs larger than L2, no flush).
              Otherwise one step per graph replay with L2 flushed by writing
              then reading 512 MiB before every step, outside its events.
              Reported beside it: the latency of one call at a time (L2
@@ -65,6 +67,11 @@ def parse():
     ap.add_argument("--replicas", type=int, default=0,
                     help="table replicas the timed steps rotate through (0: as many as keep L2 cold; "
                          "1: one table, L2 flushed before every step, e.g. for small profiler captures)")
+    ap.add_argument("--streams", type=int, default=0,
+                    help="streams the replicated steps rotate over (0: the plan's; must divide --replicas)")
+    ap.add_argument("--small-grid", type=int, default=-1,
+                    help="SMs the routing and bucketing grids are sized for in the replicated steps "
+                         "(-1: 24 with four or more streams, else all; 0: all)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle baseline")
     return ap.parse_args()
 
@@ -191,7 +198,9 @@ def aggregate_ranks(total_ms, e2e_ms, ws, n_tokens, steps, device):
 L2_BYTES = 129 << 20
 REPLICA_BUDGET = 24 << 30  # device bytes the table replicas may take
 MAX_REPLICAS = 16
-PIPE_STREAMS = 2           # batches in flight
+PIPE_STREAMS = 6           # most batches in flight (streams of the replicated steps)
+TABLE_STREAMS = 2          # streams the tables of the multi-table step alternate over
+SMALL_GRID_SMS = 24        # routing / bucketing grid with four or more batches in flight
 GRAPH_STEPS = 64           # steps per captured graph in the timed region
 
 
@@ -201,26 +210,28 @@ def table_bytes(w):
 
 
 def plan_replicas(w):
-    """How many table replicas the timed steps rotate through.
+    """How many table replicas the timed steps rotate through, and over how many streams.
 
     Each step reads about step_bytes that the previous steps did not; with R
     replicas used in turn, R - 1 other steps (at least 5x L2 of traffic) pass
     between two uses of one replica, so every step starts with its table data
-    out of L2 and no flush is needed.  R is a multiple of the stream count so
-    a replica always runs on the same stream.  Returns 1 (flush before every
-    step instead) when that many replicas do not fit the budget or the table
-    is not HBM-resident."""
+    out of L2 and no flush is needed.  The streams (batches in flight) are at
+    most PIPE_STREAMS and at most the replicas that rule asks for; R is a
+    multiple of the stream count so a replica always runs on the same stream.
+    Returns (1, 1) (flush before every step instead) when that many replicas
+    do not fit the budget or the table is not HBM-resident."""
     from paper_2607_16305_gb300 import workloads as W
 
     if w.residency != "device" or w.n_tables != 1:
-        return 1
+        return 1, 1
     d = W.expected_distinct(w.n_tokens, w.n_scenes)
     step = algorithmic_bytes(w, d, int(w.n_tokens * w.keep_ratio))["step"]
     need = 1 + math.ceil(5 * L2_BYTES / step)
-    need = ((need + PIPE_STREAMS - 1) // PIPE_STREAMS) * PIPE_STREAMS
+    ns = min(PIPE_STREAMS, need)
+    need = ((need + ns - 1) // ns) * ns
     if need > MAX_REPLICAS or need * table_bytes(w) > REPLICA_BUDGET:
-        return 1
-    return need
+        return 1, 1
+    return need, ns
 
 
 def run_lookme(args, w, ws, rank, local):
@@ -240,9 +251,15 @@ def run_lookme(args, w, ws, rank, local):
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
 
-    R = plan_replicas(w) if args.replicas <= 0 else args.replicas
-    if R > 1 and R % PIPE_STREAMS:
-        raise SystemExit(f"--replicas must be 1 or a multiple of {PIPE_STREAMS}")
+    R, NS = plan_replicas(w)
+    if args.replicas > 0:
+        R = args.replicas
+        NS = max(d for d in range(1, min(PIPE_STREAMS, R) + 1) if R % d == 0)
+    if args.streams > 0:
+        NS = args.streams
+    if R % NS:
+        raise SystemExit(f"--streams ({NS}) must divide the replicas ({R})")
+    small_grid = args.small_grid if args.small_grid >= 0 else (SMALL_GRID_SMS if NS >= 4 else 0)
     tabs = [lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=w.dtype, device=local,
                          max_tokens=w.n_tokens) for _ in range(R)]
     cent = W.centroids(w, 0, dev)
@@ -263,7 +280,11 @@ def run_lookme(args, w, ws, rank, local):
     seg = w.segment_offsets if w.n_segments > 1 else None
     flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
     flush_sink = torch.zeros((), dtype=torch.int64, device=dev)
-    streams = [torch.cuda.Stream(dev) for _ in range(PIPE_STREAMS)] if R > 1 else [stream]
+    streams = [torch.cuda.Stream(dev) for _ in range(NS)] if R > 1 else [stream]
+
+    def set_grid(sms):
+        for t in tabs:
+            t.set_small_grid(sms)
 
     def step(r, q=None, hidden=None):
         sc, pr, wt, mk = outs[r]
@@ -277,8 +298,8 @@ def run_lookme(args, w, ws, rank, local):
         flush_sink.copy_(flush.sum(dtype=torch.int64))
 
     def pipelined(n, body):
-        # Step i on replica i % R, issued on stream i % PIPE_STREAMS: two
-        # batches in flight, each replica always on the same stream.
+        # Step i on replica i % R, issued on stream i % NS: NS batches in
+        # flight, each replica always on the same stream.
         cur = torch.cuda.current_stream(dev)
         for s in streams:
             s.wait_stream(cur)
@@ -299,10 +320,13 @@ def run_lookme(args, w, ws, rank, local):
     step(0)
     torch.cuda.synchronize(dev)
     launches_per_step = tabs[0].launch_count() - c0
+    ref_out = [o.clone() for o in outs[0]]  # replica 0's results, default grids
 
     # Graphs of the steps (the library never allocates or syncs inside a call
     # once scratch is reserved).  With replicas: up to GRAPH_STEPS steps per
     # graph, pipelined over the streams; without: one step per graph.
+    if R > 1:
+        set_grid(small_grid)
     side = torch.cuda.Stream(dev)
     side.wait_stream(stream)
     with torch.cuda.stream(side):
@@ -359,9 +383,13 @@ def run_lookme(args, w, ws, rank, local):
     if ws > 1:
         dist.barrier()
     launches = launches_per_step * args.steps
+    for a, b in zip(ref_out, outs[0]):
+        if not torch.equal(a, b):
+            raise SystemExit("the timed steps' results differ from the first call's")
 
     # -------------- one call at a time: L2 flushed, one graph replay per call
     if g1 is None:
+        set_grid(0)
         g1 = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g1):
             step(0)
@@ -378,6 +406,7 @@ def run_lookme(args, w, ws, rank, local):
 
     # ---------------------- the same steps as eager C-ABI calls from Python
     if R > 1:
+        set_grid(small_grid)
         ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         ea.record(stream)
         pipelined(args.steps, step)
@@ -396,6 +425,7 @@ def run_lookme(args, w, ws, rank, local):
         eager_ms = sum(s.elapsed_time(e) for s, e in zip(estarts, eends)) / args.steps
 
     # ----------------------------------------- per-kernel durations (traced)
+    set_grid(0)
     t0 = tabs[0]
     t0.trace_enable(True)
     t0.trace_read()
@@ -433,6 +463,7 @@ def run_lookme(args, w, ws, rank, local):
             ho.copy_(hd, non_blocking=True)
 
     if R > 1:
+        set_grid(small_grid)
         xa, xb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         xa.record(stream)
         pipelined(args.steps, e2e_step)
@@ -468,8 +499,9 @@ def run_lookme(args, w, ws, rank, local):
     if R > 1:
         l2 = (f"inputs larger than L2: {R} replicas of the table ({table_bytes(w) * R / 2**30:.1f} GiB) used in turn, "
               f"{R - 1} other steps between two uses of one replica; no flush")
-        launch = (f"{PIPE_STREAMS} batches in flight: step i on replica i % {R} on stream i % {PIPE_STREAMS}; "
-                  f"{per_graph} steps per CUDA graph; one event pair around all {args.steps} steps")
+        launch = (f"{NS} batches in flight: step i on replica i % {R} on stream i % {NS}; routing and bucketing "
+                  f"grids sized for {small_grid or 'all'} SMs; {per_graph} steps per CUDA graph; one event pair "
+                  f"around all {args.steps} steps")
     else:
         l2 = f"flushed before every step ({FLUSH_BYTES >> 20} MiB written then read, outside the events)"
         launch = "step replayed as one CUDA graph (kernels chained by programmatic dependent launch)"
@@ -479,7 +511,7 @@ def run_lookme(args, w, ws, rank, local):
         "vs_baseline": None, "dtype": w.dtype, "data": "synthetic (seeded Gaussian mixture, random tables)",
         "config": {"workload": w.name, "tokens": N, "d_key": w.d_key, "scenes": w.n_scenes, "prims": w.n_prims,
                    "d_value": w.d_value, "top_k": K, "keep_ratio": w.keep_ratio, "layers": L,
-                   "replicas": R, "l2": l2, "launch": launch,
+                   "replicas": R, "streams": NS, "small_grid_sms": small_grid, "l2": l2, "launch": launch,
                    "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "kernel": "score (level-2 key scoring + top-k + softmax)",
                      "achieved": achieved, "peak": hbm, "unit": "GB/s",
@@ -543,7 +575,7 @@ def run_multitable(args, w, ws, rank, local):
     outs = [(torch.empty(N, dtype=torch.int32, device=dev), torch.empty(N, K, dtype=torch.int32, device=dev),
              torch.empty(N, K, dtype=torch.float32, device=dev), torch.empty(N, dtype=torch.uint8, device=dev))
             for _ in range(T)]
-    streams = [torch.cuda.Stream(dev) for _ in range(PIPE_STREAMS)]
+    streams = [torch.cuda.Stream(dev) for _ in range(TABLE_STREAMS)]
     flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
     flush_sink = torch.zeros((), dtype=torch.int64, device=dev)
 
@@ -645,7 +677,7 @@ def run_multitable(args, w, ws, rank, local):
                    "scenes": w.n_scenes, "prims": w.n_prims, "d_value": w.d_value, "top_k": K,
                    "keep_ratio": w.keep_ratio, "residency": "pinned host, HBM slot cache per table",
                    "l2": "cold: slot caches emptied and L2 flushed before every step, outside the events",
-                   "launch": f"one lookme_lookup_inject per table, tables alternating over {PIPE_STREAMS} streams"},
+                   "launch": f"one lookme_lookup_inject per table, tables alternating over {TABLE_STREAMS} streams"},
         "roofline": {"bound": "host link", "staged_key_bytes_per_step": staged,
                      "achieved": staged / (ms_per_step * 1e-3) / 1e9, "peak": link_gbs, "unit": "GB/s",
                      "frac": staged / (ms_per_step * 1e-3) / 1e9 / link_gbs,

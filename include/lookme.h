@@ -198,6 +198,18 @@ lookme_status lookme_reserve(lookme_table* table, int64_t max_tokens);
  * HBM-resident tables.  Errors: INVALID_ARG, CUDA. */
 lookme_status lookme_stage_invalidate(lookme_table* table, lookme_stream stream);
 
+/* Size the level-1 routing and the bucketing + gate launches of later calls
+ * for `sms` SMs instead of the whole device (0 restores the whole device).
+ * One call at a time, the default spreads these latency-bound steps over as
+ * many CTAs as there are SMs.  When several calls are in flight on different
+ * streams (Sec. "Hierarchical Lookup" over independent batches), the level-2
+ * kernel of one call holds every SM it can get, and each CTA of another call's
+ * routing or gate occupies an SM that level 2 would otherwise stream on; fewer,
+ * fuller CTAs then cost less SM time for the same work.  Results do not
+ * depend on it.  The fused single-launch form ignores it.  Not thread-safe
+ * with calls in flight on the host.  Errors: INVALID_ARG (sms < 0). */
+lookme_status lookme_set_small_grid(lookme_table* table, int32_t sms);
+
 /* Statistics of the table's most recent lookup, read back synchronously on
  * the given stream: routed scenes, level-2 work items, largest bucket. */
 typedef struct {
@@ -212,8 +224,10 @@ lookme_status lookme_last_lookup_stats(lookme_table* table, lookme_lookup_stats*
 
 /* Device status word of the table (bit 0: a bounded wait inside a kernel
  * gave up; the kernel then skipped its remaining work; bit 1: it was the
- * level-1 kernel, bit 2: a level-2 kernel).  Synchronises the stream.
- * reset != 0 clears it afterwards. */
+ * level-1 kernel, bit 2: a level-2 kernel; bit 4: more routed scenes than
+ * HBM slots; bit 6: a kernel met an index outside its range, such as an
+ * injection record naming no token, and skipped that access).  Synchronises
+ * the stream.  reset != 0 clears it afterwards. */
 lookme_status lookme_device_status(lookme_table* table, uint32_t* status, int reset, lookme_stream stream);
 
 /* Number of CUDA kernels this table has launched since creation. */

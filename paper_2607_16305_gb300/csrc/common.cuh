@@ -49,6 +49,7 @@ constexpr uint32_t STATUS_IN_ROUTE = 2u;  // set with STATUS_WAIT_TIMEOUT by the
 constexpr uint32_t STATUS_IN_SCORE = 4u;  // set with STATUS_WAIT_TIMEOUT by a level-2 kernel
 constexpr uint32_t STATUS_IN_STEP = 8u;   // set with STATUS_WAIT_TIMEOUT by the fused step kernel
 constexpr uint32_t STATUS_STAGE_OVERFLOW = 16u;  // more routed scenes than HBM slots (keys not staged)
+constexpr uint32_t STATUS_BAD_INDEX = 64u;  // a kernel met an index outside its range and skipped the access
 
 // ------------------------------------------------------------ element access
 __device__ __forceinline__ float to_f32(float x) { return x; }
@@ -261,6 +262,7 @@ struct InjectArgs {
     int64_t S;
     int n_layers;
     void* hidden[LOOKME_MAX_LAYERS];
+    uint32_t* status;     // STATUS_BAD_INDEX when a record names no token (records form)
 };
 cudaError_t launch_inject(const LaunchCtx& c, const InjectArgs& a);
 // K4 from the records the tcgen05 level-2 kernel wrote (ScoreArgs::rec_*):

@@ -72,6 +72,7 @@ struct Params {
     int64_t S;
     int n_layers;
     void* hidden[LOOKME_MAX_LAYERS];
+    uint32_t* status;
 };
 }  // namespace k4
 
@@ -277,6 +278,7 @@ cudaError_t launch_select_inject(const LaunchCtx& c, const InjectArgs& a, const 
     p.S = a.S;
     p.n_layers = a.n_layers;
     for (int l = 0; l < a.n_layers; ++l) p.hidden[l] = a.hidden[l];
+    p.status = a.status;
     k5::Params sp;
     sp.priority = priority;
     sp.mask = mask;
@@ -303,6 +305,10 @@ __global__ void __launch_bounds__(k4::kThreads) k4_inject_records(const __grid_c
     pdl_wait();
     const int64_t b = blockIdx.x;
     const int64_t t = rec_t[b];  // every thread, together with the rows and weights
+    if (t < 0 || t >= p.N) {  // a slot the level-2 kernel left unwritten: skip it (uniform for the CTA)
+        if (threadIdx.x == 0 && p.status) atomicOr(p.status, STATUS_BAD_INDEX);
+        return;
+    }
     const int j = threadIdx.x;
     if (j < p.top_k) {
         const int64_t r = min(max((int64_t)rec_row[b * p.top_k + j], (int64_t)0), p.S * p.P - 1);
@@ -330,6 +336,7 @@ cudaError_t launch_inject_records(const LaunchCtx& c, const InjectArgs& a, const
     p.S = a.S;
     p.n_layers = a.n_layers;
     for (int l = 0; l < a.n_layers; ++l) p.hidden[l] = a.hidden[l];
+    p.status = a.status;
     const int chunks = a.dv / (a.dtype == LOOKME_BF16 ? 8 : 4);
     int threads = (chunks + 31) / 32 * 32;
     if (threads > k4::kThreads) threads = k4::kThreads;
@@ -355,6 +362,7 @@ cudaError_t launch_inject(const LaunchCtx& c, const InjectArgs& a) {
     p.S = a.S;
     p.n_layers = a.n_layers;
     for (int l = 0; l < a.n_layers; ++l) p.hidden[l] = a.hidden[l];
+    p.status = a.status;
     // One 16-byte chunk of the row per thread where the row allows it.
     const int chunks = a.dv / (a.dtype == LOOKME_BF16 ? 8 : 4);
     int threads = (chunks + 31) / 32 * 32;

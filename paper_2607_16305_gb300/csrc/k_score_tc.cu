@@ -362,11 +362,15 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
                     const int64_t row = (int64_t)items[ms].scene * P + r.p;
                     if (rec_t) {
                         const int pos = tpos[ms * kTok + eg];
-                        if (lane < top_k) {
-                            rec_row[(int64_t)pos * top_k + lane] = (int32_t)row;
-                            rec_w[(int64_t)pos * top_k + lane] = r.w;
+                        if (pos < 0) {  // a kept token without a kept-list slot: skip its record
+                            if (lane == 0) atomicOr(status, STATUS_BAD_INDEX);
+                        } else {
+                            if (lane < top_k) {
+                                rec_row[(int64_t)pos * top_k + lane] = (int32_t)row;
+                                rec_w[(int64_t)pos * top_k + lane] = r.w;
+                            }
+                            if (lane == 0) rec_t[pos] = (int32_t)t;
                         }
-                        if (lane == 0) rec_t[pos] = (int32_t)t;
                     }
                     if (r.p >= 0) k3tc::prefetch_row_l2(values + row * vrow_bytes, vrow_bytes);
                     if (hidden0 && lane == 0) k3tc::prefetch_row_l2(hidden0 + t * vrow_bytes, vrow_bytes);
@@ -456,9 +460,11 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
                 }
                 return got != 0;
             };
+            // The queue barriers are thread 0's to initialise: none is touched
+            // before it has published them.
+            if (i == 0 && !__all_sync(0xFFFFFFFFu, ptx::mbar_wait(setup, 0, abort, kTimeoutNs))) break;
             have = take_next(false);
             ptx::cp_async_wait_all();
-            if (i == 0 && !__all_sync(0xFFFFFFFFu, ptx::mbar_wait(setup, 0, abort, kTimeoutNs))) break;
             ptx::fence_proxy_async_smem();  // the tile is read by the tensor core (async proxy)
             if (lane < nb) toks[ms * kTok + lane] = tok;
             const uint32_t kbits = __ballot_sync(0xFFFFFFFFu, kpos >= 0);

@@ -214,6 +214,13 @@ cudaError_t stage_invalidate(lookme_table* t, cudaStream_t s) {
     return e;
 }
 
+lookme_status lookme_set_small_grid(lookme_table* t, int32_t sms) {
+    if (!t) return fail(LOOKME_ERR_INVALID_ARG, "table is NULL");
+    if (sms < 0) return fail(LOOKME_ERR_INVALID_ARG, "sms must be >= 0 (got %d)", (int)sms);
+    t->small_sms = sms;
+    return LOOKME_OK;
+}
+
 lookme_status lookme_stage_invalidate(lookme_table* t, lookme_stream stream) {
     lookme_status st = check_table(t);
     if (st != LOOKME_OK) return st;
@@ -407,6 +414,8 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
                         nullptr, 0, nullptr);
     if ((st = ensure_scratch(t, N, s)) != LOOKME_OK) return st;
     LaunchCtx ctx{s, t->num_sms};
+    // Routing and bucketing grids: sized for small_sms SMs when it is set.
+    const LaunchCtx rctx{s, t->small_sms > 0 ? std::min(t->small_sms, t->num_sms) : t->num_sms};
     const int dk = (int)d.d_key;
     const float* bias = t->has_bias ? t->bias : nullptr;
 
@@ -419,15 +428,15 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
             return fail(LOOKME_ERR_CUDA, "cuTensorMapEncodeTiled failed for the queries");
         const void* mc[3] = {&t->tmap_c[0], &t->tmap_c[1], &t->tmap_c[2]};
         st = launch(t, s, KID_ROUTE_TC, [&] {
-            return launch_route_tc(ctx, &mq, mc, N, d.n_scenes, dk, t->inv_cnorm, bias, t->qnorm, qnorm_out, t->best,
+            return launch_route_tc(rctx, &mq, mc, N, d.n_scenes, dk, t->inv_cnorm, bias, t->qnorm, qnorm_out, t->best,
                                    t->status);
         });
     } else {
         st = launch(t, s, KID_PREP,
-                    [&] { return launch_prep(ctx, d.dtype, queries, N, dk, t->qnorm, qnorm_out, t->best); });
+                    [&] { return launch_prep(rctx, d.dtype, queries, N, dk, t->qnorm, qnorm_out, t->best); });
         if (st != LOOKME_OK) return st;
         st = launch(t, s, KID_ROUTE_SIMT, [&] {
-            return launch_route_simt(ctx, d.dtype, queries, t->cent, N, d.n_scenes, dk, t->inv_cnorm, bias, t->qnorm,
+            return launch_route_simt(rctx, d.dtype, queries, t->cent, N, d.n_scenes, dk, t->inv_cnorm, bias, t->qnorm,
                                      t->best);
         });
     }
@@ -437,21 +446,21 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
     // single-CTA sort, which is then the faster choice.
     if (N <= kBucketOneCtaTokens || gate) {
         st = launch(t, s, KID_BUCKET, [&] {
-            return launch_bucket(ctx, t->best, N, d.n_scenes, scene_out, t->item_tok, t->work, t->routed,
+            return launch_bucket(rctx, t->best, N, d.n_scenes, scene_out, t->item_tok, t->work, t->routed,
                                  t->counters, gate);
         });
     } else {
         st = launch(t, s, KID_BUCKET_COUNT, [&] {
-            return launch_bucket_count(ctx, t->best, N, d.n_scenes, scene_out, t->scene_cnt, gate);
+            return launch_bucket_count(rctx, t->best, N, d.n_scenes, scene_out, t->scene_cnt, gate);
         });
         if (st == LOOKME_OK)
             st = launch(t, s, KID_BUCKET_SCAN, [&] {
-                return launch_bucket_scan(ctx, d.n_scenes, t->scene_cnt, t->scene_pos, t->work, t->routed,
+                return launch_bucket_scan(rctx, d.n_scenes, t->scene_cnt, t->scene_pos, t->work, t->routed,
                                           t->counters);
             });
         if (st == LOOKME_OK)
             st = launch(t, s, KID_BUCKET_SCATTER, [&] {
-                return launch_bucket_scatter(ctx, t->best, N, scene_out, t->scene_pos, t->item_tok);
+                return launch_bucket_scatter(rctx, t->best, N, scene_out, t->scene_pos, t->item_tok);
             });
     }
     if (st != LOOKME_OK) return st;
@@ -572,6 +581,7 @@ InjectArgs inject_args(const lookme_table* t, const int32_t* scene, const int32_
     a.S = d.n_scenes;
     a.n_layers = n_layers;
     for (int l = 0; l < n_layers; ++l) a.hidden[l] = hidden[l];
+    a.status = t->status;
     return a;
 }
 
