@@ -305,10 +305,6 @@ __global__ void __launch_bounds__(k4::kThreads) k4_inject_records(const __grid_c
     pdl_wait();
     const int64_t b = blockIdx.x;
     const int64_t t = rec_t[b];  // every thread, together with the rows and weights
-    if (t < 0 || t >= p.N) {  // a slot the level-2 kernel left unwritten: skip it (uniform for the CTA)
-        if (threadIdx.x == 0 && p.status) atomicOr(p.status, STATUS_BAD_INDEX);
-        return;
-    }
     const int j = threadIdx.x;
     if (j < p.top_k) {
         const int64_t r = min(max((int64_t)rec_row[b * p.top_k + j], (int64_t)0), p.S * p.P - 1);
@@ -316,6 +312,10 @@ __global__ void __launch_bounds__(k4::kThreads) k4_inject_records(const __grid_c
         w[j] = rec_w[b * p.top_k + j];
     }
     __syncthreads();
+    if (t < 0 || t >= p.N) {  // a slot the level-2 kernel left unwritten: skip it (uniform for the CTA)
+        if (threadIdx.x == 0 && p.status) atomicOr(p.status, STATUS_BAD_INDEX);
+        return;
+    }
     accumulate_store<T>(p, t, rows, w);
 }
 
