@@ -13,7 +13,7 @@ keep 25%) unless --workload says otherwise.
              rotate over S streams (single image: 6), so S batches are in
              flight (some batches' routing, bucketing and injection beside
              another's level 2), with the routing and bucketing grids sized
-             for 24 SMs (lookme_set_small_grid); the steps are replayed as CUDA
+             for 16 SMs (lookme_set_small_grid); the steps are replayed as CUDA
              graphs of 64 steps between one pair of events, and R - 1 other
              steps pass between two uses of a replica, so its data is out of
              L2 (inputs larger than L2, no flush).
@@ -71,7 +71,7 @@ def parse():
                     help="streams the replicated steps rotate over (0: the plan's; must divide --replicas)")
     ap.add_argument("--small-grid", type=int, default=-1,
                     help="SMs the routing and bucketing grids are sized for in the replicated steps "
-                         "(-1: 24 with four or more streams, else all; 0: all)")
+                         "(-1: 16 with four or more streams, else all; 0: all)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle baseline")
     return ap.parse_args()
 
@@ -200,7 +200,7 @@ REPLICA_BUDGET = 24 << 30  # device bytes the table replicas may take
 MAX_REPLICAS = 16
 PIPE_STREAMS = 6           # most batches in flight (streams of the replicated steps)
 TABLE_STREAMS = 2          # streams the tables of the multi-table step alternate over
-SMALL_GRID_SMS = 24        # routing / bucketing grid with four or more batches in flight
+SMALL_GRID_SMS = 16        # routing / bucketing grid with four or more batches in flight
 GRAPH_STEPS = 64           # steps per captured graph in the timed region
 
 
