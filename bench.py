@@ -9,14 +9,14 @@ keep 25%) unless --workload says otherwise.
 
   value      tokens/s over K device-timed steps, inputs resident in HBM.  When
              the table is small enough to hold several copies (single image:
-             12 replicas, 13.6 GiB), step i runs on replica i % R and the steps
-             rotate over S streams (single image: 6), so S batches are in
+             16 replicas, 18 GiB), step i runs on replica i % R and the steps
+             rotate over S streams (single image: 16), so S batches are in
              flight (some batches' routing, bucketing and injection beside
-             another's level 2), with the routing and bucketing grids sized
-             for 16 SMs (lookme_set_small_grid); the steps are replayed as CUDA
-             graphs of 64 steps between one pair of events, and R - 1 other
-             steps pass between two uses of a replica, so its data is out of
-             L2 (inputs larger than L2, no flush).
+             others' level 2), with the routing and bucketing grids sized for
+             16 SMs and level 2 on 56 CTAs (lookme_set_grids); the steps are
+             replayed as CUDA graphs of 64 steps between one pair of events,
+             and R - 1 other steps pass between two uses of a replica, so its
+             data is out of L2 (inputs larger than L2, no flush).
              Otherwise one step per graph replay with L2 flushed by writing
              then reading 512 MiB before every step, outside its events.
              Reported beside it: the latency of one call at a time (L2
@@ -72,6 +72,9 @@ def parse():
     ap.add_argument("--small-grid", type=int, default=-1,
                     help="SMs the routing and bucketing grids are sized for in the replicated steps "
                          "(-1: 16 with four or more streams, else all; 0: all)")
+    ap.add_argument("--level2-ctas", type=int, default=-1,
+                    help="CTAs of level 2 in the replicated steps (-1: 56 with four or more streams, else one "
+                         "per SM; 0: one per SM)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle baseline")
     return ap.parse_args()
 
@@ -198,9 +201,10 @@ def aggregate_ranks(total_ms, e2e_ms, ws, n_tokens, steps, device):
 L2_BYTES = 129 << 20
 REPLICA_BUDGET = 24 << 30  # device bytes the table replicas may take
 MAX_REPLICAS = 16
-PIPE_STREAMS = 6           # most batches in flight (streams of the replicated steps)
+PIPE_STREAMS = 16          # most batches in flight (streams of the replicated steps)
 TABLE_STREAMS = 2          # streams the tables of the multi-table step alternate over
 SMALL_GRID_SMS = 16        # routing / bucketing grid with four or more batches in flight
+LEVEL2_CTAS = 56           # level-2 CTAs with four or more batches in flight
 GRAPH_STEPS = 64           # steps per captured graph in the timed region
 
 
@@ -215,11 +219,11 @@ def plan_replicas(w):
     Each step reads about step_bytes that the previous steps did not; with R
     replicas used in turn, R - 1 other steps (at least 5x L2 of traffic) pass
     between two uses of one replica, so every step starts with its table data
-    out of L2 and no flush is needed.  The streams (batches in flight) are at
-    most PIPE_STREAMS and at most the replicas that rule asks for; R is a
-    multiple of the stream count so a replica always runs on the same stream.
-    Returns (1, 1) (flush before every step instead) when that many replicas
-    do not fit the budget or the table is not HBM-resident."""
+    out of L2 and no flush is needed.  Within the budget R grows to
+    PIPE_STREAMS, one stream (batch in flight) per replica; a table that fits
+    fewer copies keeps what the rule asks for, over as many streams.  Returns
+    (1, 1) (flush before every step instead) when that many replicas do not fit
+    the budget or the table is not HBM-resident."""
     from paper_2607_16305_gb300 import workloads as W
 
     if w.residency != "device" or w.n_tables != 1:
@@ -227,11 +231,11 @@ def plan_replicas(w):
     d = W.expected_distinct(w.n_tokens, w.n_scenes)
     step = algorithmic_bytes(w, d, int(w.n_tokens * w.keep_ratio))["step"]
     need = 1 + math.ceil(5 * L2_BYTES / step)
-    ns = min(PIPE_STREAMS, need)
-    need = ((need + ns - 1) // ns) * ns
-    if need > MAX_REPLICAS or need * table_bytes(w) > REPLICA_BUDGET:
+    fit = min(MAX_REPLICAS, REPLICA_BUDGET // table_bytes(w))
+    if need > fit:
         return 1, 1
-    return need, ns
+    r = max(need, min(PIPE_STREAMS, fit))
+    return r, min(r, PIPE_STREAMS) if r % min(r, PIPE_STREAMS) == 0 else 1
 
 
 def run_lookme(args, w, ws, rank, local):
@@ -260,6 +264,7 @@ def run_lookme(args, w, ws, rank, local):
     if R % NS:
         raise SystemExit(f"--streams ({NS}) must divide the replicas ({R})")
     small_grid = args.small_grid if args.small_grid >= 0 else (SMALL_GRID_SMS if NS >= 4 else 0)
+    level2_ctas = args.level2_ctas if args.level2_ctas >= 0 else (LEVEL2_CTAS if NS >= 4 else 0)
     tabs = [lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=w.dtype, device=local,
                          max_tokens=w.n_tokens) for _ in range(R)]
     cent = W.centroids(w, 0, dev)
@@ -282,9 +287,9 @@ def run_lookme(args, w, ws, rank, local):
     flush_sink = torch.zeros((), dtype=torch.int64, device=dev)
     streams = [torch.cuda.Stream(dev) for _ in range(NS)] if R > 1 else [stream]
 
-    def set_grid(sms):
+    def set_grid(on):
         for t in tabs:
-            t.set_small_grid(sms)
+            t.set_grids(small_grid if on else 0, level2_ctas if on else 0)
 
     def step(r, q=None, hidden=None):
         sc, pr, wt, mk = outs[r]
@@ -326,7 +331,7 @@ def run_lookme(args, w, ws, rank, local):
     # once scratch is reserved).  With replicas: up to GRAPH_STEPS steps per
     # graph, pipelined over the streams; without: one step per graph.
     if R > 1:
-        set_grid(small_grid)
+        set_grid(True)
     side = torch.cuda.Stream(dev)
     side.wait_stream(stream)
     with torch.cuda.stream(side):
@@ -389,7 +394,7 @@ def run_lookme(args, w, ws, rank, local):
 
     # -------------- one call at a time: L2 flushed, one graph replay per call
     if g1 is None:
-        set_grid(0)
+        set_grid(False)
         g1 = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g1):
             step(0)
@@ -406,7 +411,7 @@ def run_lookme(args, w, ws, rank, local):
 
     # ---------------------- the same steps as eager C-ABI calls from Python
     if R > 1:
-        set_grid(small_grid)
+        set_grid(True)
         ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         ea.record(stream)
         pipelined(args.steps, step)
@@ -425,7 +430,7 @@ def run_lookme(args, w, ws, rank, local):
         eager_ms = sum(s.elapsed_time(e) for s, e in zip(estarts, eends)) / args.steps
 
     # ----------------------------------------- per-kernel durations (traced)
-    set_grid(0)
+    set_grid(False)
     t0 = tabs[0]
     t0.trace_enable(True)
     t0.trace_read()
@@ -463,7 +468,7 @@ def run_lookme(args, w, ws, rank, local):
             ho.copy_(hd, non_blocking=True)
 
     if R > 1:
-        set_grid(small_grid)
+        set_grid(True)
         xa, xb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         xa.record(stream)
         pipelined(args.steps, e2e_step)
@@ -500,8 +505,8 @@ def run_lookme(args, w, ws, rank, local):
         l2 = (f"inputs larger than L2: {R} replicas of the table ({table_bytes(w) * R / 2**30:.1f} GiB) used in turn, "
               f"{R - 1} other steps between two uses of one replica; no flush")
         launch = (f"{NS} batches in flight: step i on replica i % {R} on stream i % {NS}; routing and bucketing "
-                  f"grids sized for {small_grid or 'all'} SMs; {per_graph} steps per CUDA graph; one event pair "
-                  f"around all {args.steps} steps")
+                  f"grids sized for {small_grid or 'all'} SMs, level 2 on {level2_ctas or 'one CTA per SM'} CTAs; "
+                  f"{per_graph} steps per CUDA graph; one event pair around all {args.steps} steps")
     else:
         l2 = f"flushed before every step ({FLUSH_BYTES >> 20} MiB written then read, outside the events)"
         launch = "step replayed as one CUDA graph (kernels chained by programmatic dependent launch)"
@@ -511,7 +516,8 @@ def run_lookme(args, w, ws, rank, local):
         "vs_baseline": None, "dtype": w.dtype, "data": "synthetic (seeded Gaussian mixture, random tables)",
         "config": {"workload": w.name, "tokens": N, "d_key": w.d_key, "scenes": w.n_scenes, "prims": w.n_prims,
                    "d_value": w.d_value, "top_k": K, "keep_ratio": w.keep_ratio, "layers": L,
-                   "replicas": R, "streams": NS, "small_grid_sms": small_grid, "l2": l2, "launch": launch,
+                   "replicas": R, "streams": NS, "small_grid_sms": small_grid, "level2_ctas": level2_ctas, "l2": l2,
+                   "launch": launch,
                    "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "kernel": "score (level-2 key scoring + top-k + softmax)",
                      "achieved": achieved, "peak": hbm, "unit": "GB/s",

@@ -198,17 +198,20 @@ lookme_status lookme_reserve(lookme_table* table, int64_t max_tokens);
  * HBM-resident tables.  Errors: INVALID_ARG, CUDA. */
 lookme_status lookme_stage_invalidate(lookme_table* table, lookme_stream stream);
 
-/* Size the level-1 routing and the bucketing + gate launches of later calls
- * for `sms` SMs instead of the whole device (0 restores the whole device).
- * One call at a time, the default spreads these latency-bound steps over as
- * many CTAs as there are SMs.  When several calls are in flight on different
- * streams (Sec. "Hierarchical Lookup" over independent batches), the level-2
- * kernel of one call holds every SM it can get, and each CTA of another call's
- * routing or gate occupies an SM that level 2 would otherwise stream on; fewer,
- * fuller CTAs then cost less SM time for the same work.  Results do not
- * depend on it.  The fused single-launch form ignores it.  Not thread-safe
- * with calls in flight on the host.  Errors: INVALID_ARG (sms < 0). */
-lookme_status lookme_set_small_grid(lookme_table* table, int32_t sms);
+/* Grid sizes of later calls, for running several calls at once (Sec.
+ * "Hierarchical Lookup" over independent batches on different streams).
+ * route_sms: the SM count that the level-1 routing and the bucketing + gate
+ * size their grids for (0: the whole device).  level2_ctas: the CTAs of the
+ * tcgen05 level-2 kernel (0: one per SM; values above the SM count act as 0).
+ * One call at a time, the defaults spread every step over the whole device.
+ * With several calls in flight, each CTA of one call's routing or gate holds an
+ * SM that another call's level 2 would stream on, and each level-2 CTA pays a
+ * ramp (first copy) and a tail (last item's top-k) per call; fewer, fuller
+ * CTAs then cost less SM time for the same work, while the calls in flight
+ * together keep HBM busy.  Results do not depend on either value.  The fused
+ * single-launch form ignores both.  Not thread-safe with calls in flight on
+ * the host.  Errors: INVALID_ARG (a negative value). */
+lookme_status lookme_set_grids(lookme_table* table, int32_t route_sms, int32_t level2_ctas);
 
 /* Statistics of the table's most recent lookup, read back synchronously on
  * the given stream: routed scenes, level-2 work items, largest bucket. */

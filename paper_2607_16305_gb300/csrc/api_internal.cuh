@@ -102,6 +102,7 @@ struct lookme_table {
     size_t esz = 2;
     int num_sms = 0;
     int small_sms = 0;      // SMs the routing and bucketing grids are sized for (0: num_sms)
+    int level2_ctas = 0;    // CTAs of the tcgen05 level 2 (0: num_sms)
     bool tc_route = false;  // level 1 on tcgen05
     bool tc_score = false;  // level 2 on tcgen05
     bool use_step = false;  // whole calls as one fused launch where the shape allows

@@ -214,10 +214,12 @@ cudaError_t stage_invalidate(lookme_table* t, cudaStream_t s) {
     return e;
 }
 
-lookme_status lookme_set_small_grid(lookme_table* t, int32_t sms) {
+lookme_status lookme_set_grids(lookme_table* t, int32_t route_sms, int32_t level2_ctas) {
     if (!t) return fail(LOOKME_ERR_INVALID_ARG, "table is NULL");
-    if (sms < 0) return fail(LOOKME_ERR_INVALID_ARG, "sms must be >= 0 (got %d)", (int)sms);
-    t->small_sms = sms;
+    if (route_sms < 0 || level2_ctas < 0)
+        return fail(LOOKME_ERR_INVALID_ARG, "grid sizes must be >= 0 (got %d, %d)", (int)route_sms, (int)level2_ctas);
+    t->small_sms = route_sms;
+    t->level2_ctas = level2_ctas;
     return LOOKME_OK;
 }
 
@@ -513,7 +515,12 @@ lookme_status lookup_impl(lookme_table* t, const void* queries, int64_t N, int32
     a.rec_row = gated && records ? t->rec_row : nullptr;
     a.rec_w = gated && records ? t->rec_w : nullptr;
     st = launch(t, s, KID_SCORE,
-                [&] { return t->tc_score ? launch_score_tc(ctx, a.keys, a) : launch_score(ctx, a); });
+                [&] {
+                    if (!t->tc_score) return launch_score(ctx, a);
+                    // The level-2 grid: level2_ctas CTAs when it is set.
+                    const LaunchCtx lctx{s, t->level2_ctas > 0 ? std::min(t->level2_ctas, t->num_sms) : t->num_sms};
+                    return launch_score_tc(lctx, a.keys, a);
+                });
     if (st != LOOKME_OK) return st;
     t->last_tokens = N;
     return LOOKME_OK;

@@ -24,7 +24,7 @@ ROUTE_STATIC_MAX_TOKENS = 65536
 
 EXPORTS = [
     "lookme_table_create", "lookme_table_destroy", "lookme_load_scenes", "lookme_lookup", "lookme_inject",
-    "lookme_reserve", "lookme_stage_invalidate", "lookme_set_small_grid", "lookme_last_lookup_stats", "lookme_device_status", "lookme_launch_count",
+    "lookme_reserve", "lookme_stage_invalidate", "lookme_set_grids", "lookme_last_lookup_stats", "lookme_device_status", "lookme_launch_count",
     "lookme_trace_enable", "lookme_trace_read", "lookme_kernel_name", "lookme_status_string",
     "lookme_last_error", "lookme_route_scenes_static", "lookme_lookup_inject",
     "lookme_set_ranker", "lookme_lookup_ranked", "lookme_ska_gate", "lookme_inject_gated", "lookme_combine",
@@ -78,7 +78,7 @@ def load(path: str = LIB_PATH):
         "lookme_inject": ([P, P, P, P, I64, I32, P, P, I32, D, P, I32, P, P, P], I32),
         "lookme_reserve": ([P, I64], I32),
         "lookme_stage_invalidate": ([P, P], I32),
-        "lookme_set_small_grid": ([P, I32], I32),
+        "lookme_set_grids": ([P, I32, I32], I32),
         "lookme_last_lookup_stats": ([P, ctypes.POINTER(LookupStats), P], I32),
         "lookme_device_status": ([P, ctypes.POINTER(ctypes.c_uint32), I32, P], I32),
         "lookme_launch_count": ([P], ctypes.c_uint64),
@@ -263,9 +263,10 @@ class Table:
         """Empty the HBM slot cache of a pinned-host table (the next lookup copies every routed scene)."""
         _check(self.lib.lookme_stage_invalidate(self.handle, _stream(stream, self.device)))
 
-    def set_small_grid(self, sms):
-        """Size the routing and bucketing grids of later calls for `sms` SMs (0: all of them)."""
-        _check(self.lib.lookme_set_small_grid(self.handle, int(sms)))
+    def set_grids(self, route_sms=0, level2_ctas=0):
+        """Grid sizes of later calls: routing and bucketing for `route_sms` SMs, level 2 on
+        `level2_ctas` CTAs (0: the whole device)."""
+        _check(self.lib.lookme_set_grids(self.handle, int(route_sms), int(level2_ctas)))
 
     def device_status(self, reset=False, stream=None):
         v = ctypes.c_uint32()

@@ -22,12 +22,12 @@ def _bias(w, scale, seed=11):
 
 
 def run_case(o, lookme_lib, w, *, sample=None, give_centroids=True, bias_scale=0.0, n_layers=None,
-             residency=None, table=0, mu=None, report=None, with_sel=False, fused=False, small_grid=0):
+             residency=None, table=0, mu=None, report=None, with_sel=False, fused=False, grids=(0, 0)):
     """with_sel requests the kept-id list, which routes the injection through
     the separate selection kernel; without it short segments take the fused
     select + inject kernel.  fused uses lookme_lookup_inject instead of the
-    two calls.  small_grid sizes the routing and bucketing grids for that
-    many SMs (lookme_set_small_grid)."""
+    two calls.  grids = (routing and bucketing SMs, level-2 CTAs) for
+    lookme_set_grids (0: the whole device)."""
     from paper_2607_16305_gb300 import lookme
 
     L = n_layers or w.layers_per_table
@@ -37,7 +37,7 @@ def run_case(o, lookme_lib, w, *, sample=None, give_centroids=True, bias_scale=0
     with lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=w.dtype,
                       residency=residency or w.residency, device=0) as t:
         cent = H.load_table(t, w, table, DEV, mu, give_centroids, bias)
-        t.set_small_grid(small_grid)
+        t.set_grids(*grids)
         q = W.queries(w, DEV, mu)
         hs = [W.hidden(w, l, DEV) for l in range(L)]
         h0 = [h.clone() for h in hs]
