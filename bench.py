@@ -759,7 +759,7 @@ def run_path(args, w):
     sampler = ClockSampler(0)
     sampler.start()
     if args.path == "ranked":
-        dm, R = 256, 10  # 10 table replicas (11.3 GiB) for the two-stream measurement, as for the keys path
+        dm, R = 256, PIPE_STREAMS  # one table replica per batch in flight, as for the keys path
         W1, b1 = rnd((dm, 2 * w.d_key), 1, 1 / math.sqrt(2 * w.d_key)), rnd((dm,), 2, 0.1, torch.float32)
         W2, b2 = rnd((w.n_prims, dm), 3, 2 / math.sqrt(dm)), rnd((w.n_prims,), 4, 0.1, torch.float32)
         tabs = [lookme.Table(w.n_scenes, w.n_prims, w.d_key, w.d_value, dtype=w.dtype, device=0, max_tokens=N)
@@ -799,15 +799,18 @@ def run_path(args, w):
         torch.cuda.synchronize()
         launches = t.launch_count() - c0 + 1  # + the gate kernel (table-less)
         latency_ms = _time_calls(fn, args.steps, args.warmup, flush, stream)
-        # Two batches in flight over the replicas (graphs of 64 steps), as the keys path's value.
-        streams = [torch.cuda.Stream(dev) for _ in range(2)]
+        # Batches in flight over the replicas, one stream each (graphs of 64 steps), with the routing
+        # grid sized for SMALL_GRID_SMS SMs, as the keys path's value.
+        for t_ in tabs:
+            t_.set_grids(SMALL_GRID_SMS, 0)
+        streams = [torch.cuda.Stream(dev) for _ in range(R)]
         gph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(gph):
             cur = torch.cuda.current_stream(dev)
             for s_ in streams:
                 s_.wait_stream(cur)
             for i in range(64):
-                with torch.cuda.stream(streams[i % 2]):
+                with torch.cuda.stream(streams[i % R]):
                     fn_r(i % R)
             for s_ in streams:
                 cur.wait_stream(s_)
@@ -822,6 +825,7 @@ def run_path(args, w):
         eb.record(stream)
         torch.cuda.synchronize()
         ms = ea.elapsed_time(eb) / (reps * 64)
+        t.set_grids(0, 0)
         t.trace_enable(True)
         t.trace_read()
         _time_calls(fn, min(args.steps, 50), 1, flush, stream)
