@@ -55,14 +55,18 @@ def test_duplicated_centroids_route_to_the_lower_scene(oracle, lookme_lib, path)
     assert (r["scene"][tied] == 4).all() and (gs[tied] == 4).all()
 
 
-def test_equal_keys_take_the_lower_primitives(lookme_lib, path):
+@pytest.mark.parametrize("n_prims", [64, 512])
+def test_equal_keys_take_the_lower_primitives(lookme_lib, path, n_prims):
     """Scene 2: every key equal, so every logit ties and the top-k is
     primitives 0..k-1 in that order, each weighted exactly 1/k.  Scene 1: keys
     repeat with period 4, so the top-8 is the eight lowest members of the best
-    of the four groups, in increasing order, each weighted 1/8."""
+    of the four groups, in increasing order, each weighted 1/8.  With 512
+    primitives the logits come from two N-tiles, and the equal keys of the
+    second must not displace the lower ones of the first."""
     from paper_2607_16305_gb300 import lookme
 
-    w = W.small("tie_prim", n_tokens=800, n_scenes=4, n_prims=64, d_key=64, d_value=32, top_k=8, keep_ratio=0.25)
+    w = W.small(f"tie_prim_{n_prims}", n_tokens=800, n_scenes=4, n_prims=n_prims, d_key=64, d_value=32, top_k=8,
+                keep_ratio=0.25)
     cent, keys, vals = W.full_table(w, device=DEV)
     keys[2] = keys[2, 0:1].expand(w.n_prims, -1)
     keys[1] = keys[1, 0:4].repeat(w.n_prims // 4, 1)
