@@ -23,7 +23,8 @@ keep 25%) unless --workload says otherwise.
              flushed, one graph replay) and the eager time.
   e2e        the same through host buffers: pinned-host queries and hidden
              states copied in and the updated hidden states copied out, inside
-             the timed region
+             the timed region, every step (replayed from the same kind of CUDA
+             graphs as value when the steps are replicated)
   roofline   the level-2 scoring kernel (the dominant one): algorithmic bytes
              per launch / its mean event-timed duration, against the measured
              HBM copy bandwidth
@@ -468,10 +469,31 @@ def run_lookme(args, w, ws, rank, local):
             ho.copy_(hd, non_blocking=True)
 
     if R > 1:
+        # The same graphs of GRAPH_STEPS steps as the timed value, each step with
+        # its copies in and out (captured as copy nodes from and to pinned host
+        # memory), so the host-side launch cost of one call per step does not
+        # stand in for the link.
         set_grid(True)
+        for r in range(R):
+            e2e_step(r)
+        torch.cuda.synchronize(dev)
+
+        def capture_e2e(n):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                pipelined(n, e2e_step)
+            return g
+
+        ge_full = capture_e2e(per_graph)
+        ge_rem = capture_e2e(args.steps % per_graph) if args.steps % per_graph else None
+        ge_full.replay()
+        torch.cuda.synchronize(dev)
         xa, xb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         xa.record(stream)
-        pipelined(args.steps, e2e_step)
+        for _ in range(args.steps // per_graph):
+            ge_full.replay()
+        if ge_rem is not None:
+            ge_rem.replay()
         xb.record(stream)
         torch.cuda.synchronize(dev)
         e2e_ms = xa.elapsed_time(xb)
@@ -533,7 +555,8 @@ def run_lookme(args, w, ws, rank, local):
         "kernels_ms": kernels_ms, "traced_ms_per_step": traced_ms / args.steps,
         "routed_scenes": stats["n_routed_scenes"], "selected_tokens": n_sel,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "ms_per_step": e2e_ms / args.steps},
+                "ms_per_step": e2e_ms / args.steps,
+                "launch": "CUDA graphs of the steps with their copies" if R > 1 else "one eager call per step"},
         "gpu_launches": launches,
         "clocks": clocks,
     }
