@@ -732,19 +732,31 @@ def run_multitable(args, w, ws, rank, local):
 PATHS = ("ranked", "fusion", "router", "project", "text")
 
 
-def _time_calls(fn, steps, warmup, flush, stream, sampler=None):
+def _time_calls(fn, steps, warmup, flush, stream, sampler=None, graph=True):
+    """Mean device time of one call of fn, L2 flushed before each, events
+    around each.  graph: the call is captured once as a CUDA graph and
+    replayed, so the host's argument marshalling and launch work of an eager
+    call (which the events would otherwise bracket while the GPU waits) is
+    left out."""
     import torch
 
     for i in range(warmup):
         flush(i)
         fn()
     torch.cuda.synchronize()
+    run = fn
+    if graph:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            fn()
+        torch.cuda.synchronize()
+        run = g.replay
     st = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     en = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     for i in range(steps):
         flush(i)
         st[i].record(stream)
-        fn()
+        run()
         en[i].record(stream)
     torch.cuda.synchronize()
     return statistics.mean(a.elapsed_time(b) for a, b in zip(st, en))
@@ -851,7 +863,7 @@ def run_path(args, w):
         t.set_grids(0, 0)
         t.trace_enable(True)
         t.trace_read()
-        _time_calls(fn, min(args.steps, 50), 1, flush, stream)
+        _time_calls(fn, min(args.steps, 50), 1, flush, stream, graph=False)
         for name, v in t.trace_read(max_records=2000):
             kernels.setdefault(name, []).append(v)
         t.trace_enable(False)
