@@ -209,8 +209,9 @@ lookme_status lookme_stage_invalidate(lookme_table* table, lookme_stream stream)
  * ramp (first copy) and a tail (last item's top-k) per call; fewer, fuller
  * CTAs then cost less SM time for the same work, while the calls in flight
  * together keep HBM busy.  Results do not depend on either value.  The fused
- * single-launch form ignores both.  Not thread-safe with calls in flight on
- * the host.  Errors: INVALID_ARG (a negative value). */
+ * single-launch form ignores both.  lookme_lookup_ranked takes route_sms for
+ * its routing grid and its ranker GEMM tiles.  Not thread-safe with calls in
+ * flight on the host.  Errors: INVALID_ARG (a negative value). */
 lookme_status lookme_set_grids(lookme_table* table, int32_t route_sms, int32_t level2_ctas);
 
 /* Statistics of the table's most recent lookup, read back synchronously on

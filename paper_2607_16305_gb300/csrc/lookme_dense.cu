@@ -149,6 +149,9 @@ lookme_status lookme_lookup_ranked(lookme_table* t, const void* queries, int64_t
     if ((st = ensure_scratch(t, N, s)) != LOOKME_OK) return st;
     if ((st = ensure_ranker_scratch(t, N, s)) != LOOKME_OK) return st;
     LaunchCtx ctx{s, t->num_sms};
+    // lookme_set_grids: the routing grid and the GEMM tiles sized for route_sms SMs.
+    const int gsms = t->small_sms > 0 ? std::min(t->small_sms, t->num_sms) : t->num_sms;
+    const LaunchCtx rctx{s, gsms};
     const int dk = (int)d.d_key;
     const float* bias = t->has_bias ? t->bias : nullptr;
     const int64_t dm = t->rk_dm, P = d.n_prims, ld_r = round_up(P, 4);
@@ -162,15 +165,15 @@ lookme_status lookme_lookup_ranked(lookme_table* t, const void* queries, int64_t
             return fail(LOOKME_ERR_CUDA, "cuTensorMapEncodeTiled failed for the queries");
         const void* mc[3] = {&t->tmap_c[0], &t->tmap_c[1], &t->tmap_c[2]};
         st = launch(t, s, KID_ROUTE_TC, [&] {
-            return launch_route_tc(ctx, &mq, mc, N, d.n_scenes, dk, t->inv_cnorm, bias, t->qnorm, nullptr, t->best,
+            return launch_route_tc(rctx, &mq, mc, N, d.n_scenes, dk, t->inv_cnorm, bias, t->qnorm, nullptr, t->best,
                                    t->status);
         });
     } else {
         st = launch(t, s, KID_PREP,
-                    [&] { return launch_prep(ctx, d.dtype, queries, N, dk, t->qnorm, nullptr, t->best); });
+                    [&] { return launch_prep(rctx, d.dtype, queries, N, dk, t->qnorm, nullptr, t->best); });
         if (st == LOOKME_OK)
             st = launch(t, s, KID_ROUTE_SIMT, [&] {
-                return launch_route_simt(ctx, d.dtype, queries, t->cent, N, d.n_scenes, dk, t->inv_cnorm, bias,
+                return launch_route_simt(rctx, d.dtype, queries, t->cent, N, d.n_scenes, dk, t->inv_cnorm, bias,
                                          t->qnorm, t->best);
             });
     }
@@ -192,12 +195,12 @@ lookme_status lookme_lookup_ranked(lookme_table* t, const void* queries, int64_t
         g.rowsel = scene_out;
         g.ld_rowbias = dm;
         g.act = 1;
-        if ((st = gemm(t, s, t->num_sms, queries, t->rk_w1v, N, dm, dk, g)) != LOOKME_OK) return st;
+        if ((st = gemm(t, s, gsms, queries, t->rk_w1v, N, dm, dk, g)) != LOOKME_OK) return st;
     }
     {
         GemmArgs g = gemm_args(EPI_F32, r, ld_r, t->status);
         g.colbias = t->rk_b2;
-        if ((st = gemm(t, s, t->num_sms, H, t->rk_w2, N, P, dm, g)) != LOOKME_OK) return st;
+        if ((st = gemm(t, s, gsms, H, t->rk_w2, N, P, dm, g)) != LOOKME_OK) return st;
     }
     // Top-T by r and the cos + tanh softmax, reading only the selected key rows.
     KeyView kv;

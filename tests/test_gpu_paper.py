@@ -106,6 +106,13 @@ def test_lookup_ranked(oracle, lookme_lib, paper_oracle, name, kw, dm):
         s2, p2, w2 = t.lookup_ranked(q, w.top_k)
         torch.cuda.synchronize()
         assert torch.equal(scene, s2) and torch.equal(prim, p2) and torch.equal(weight, w2)
+        # Routing grid and GEMM tiles for fewer SMs (lookme_set_grids): the same results.
+        for grids in ((16, 0), (1, 0)):
+            t.set_grids(*grids)
+            s3, p3, w3 = t.lookup_ranked(q, w.top_k)
+            torch.cuda.synchronize()
+            assert torch.equal(scene, s3) and torch.equal(prim, p3) and torch.equal(weight, w3), grids
+        t.set_grids(0, 0)
     qs, cent_np = H.f32(q), H.f32(cent)
     gscene, gprim, gw = scene.cpu().numpy(), prim.cpu().numpy(), weight.cpu().numpy()
     r = oracle.route(qs, cent_np)
