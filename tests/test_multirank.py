@@ -71,3 +71,19 @@ def test_reference_arm_other_ranks_exit_without_work():
                        capture_output=True, text=True, env=env, timeout=300, cwd=ROOT)
     assert r.returncode == 0, r.stderr
     assert r.stdout.strip() == ""
+
+
+def test_replica_plan():
+    """The bench's replica plan: the single image gets one table replica per
+    stream (sixteen), the batched table two, and tables that cannot be held
+    several times (or are not HBM-resident) one with L2 flushed."""
+    import bench
+    from paper_2607_16305_gb300 import workloads as W
+
+    assert bench.plan_replicas(W.WORKLOADS["single_image"]) == (16, 16)
+    assert bench.plan_replicas(W.WORKLOADS["batched_zipf"]) == (2, 2)
+    assert bench.plan_replicas(W.WORKLOADS["large_table"]) == (1, 1)
+    assert bench.plan_replicas(W.WORKLOADS["multilayer_host"]) == (1, 1)
+    for w in W.WORKLOADS.values():
+        r, ns = bench.plan_replicas(w)
+        assert r % ns == 0 and r * bench.table_bytes(w) <= max(bench.REPLICA_BUDGET, bench.table_bytes(w))
