@@ -26,7 +26,7 @@ constexpr int kEpiWarps = 2 * kGroupWarps;
 constexpr int kBuildWarp = 2 + kEpiWarps;
 constexpr int kThreads = (3 + kEpiWarps) * 32;
 constexpr int kMaxStages = 14;           // ring slots (barrier arrays)
-constexpr int kBSlots = 2;               // token tiles
+constexpr int kBSlots = 3;               // token tiles
 constexpr int kISlots = 4;               // item metadata (scene, count, token ids)
 constexpr int kSeq = 4;                  // item indices passed from the producer to the token-tile warp
 constexpr uint64_t kTimeoutNs = 1000000000ull;
