@@ -38,9 +38,12 @@
 //                rows with 16-byte cp.async straight into the swizzled tile,
 //                all of them in flight at once (bulk copies of a row would
 //                each cost the copy engine as much time as a 64 KiB one)
-// Before the grid dependency wait, the MMA issuer and the top-k run once
-// without effect, so their code is cached before the key stream starts (a
-// first instruction fetch under the full stream costs microseconds).
+// Before the grid dependency wait, the MMA issuer and the second epilogue
+// group's top-k run once without effect, so their code is cached before the
+// key stream starts (a first instruction fetch under the full stream costs
+// microseconds; after an L2 flush the warm-up takes about 10 us).  The first
+// group skips it: it reads out the CTA's first item as soon as its products
+// are done, so the D buffers are not all held until the warm-up ends.
 // Every wait is bounded; on a timeout the kernel drains its copies and MMAs,
 // releases TMEM and reports through the status word.
 #include <cuda.h>
@@ -104,10 +107,11 @@ __global__ void __launch_bounds__(k3tc::kThreads, 1)
         ptx::fence_mbar_init();
     }
     __syncthreads();
-    // Warm-up while the predecessor finishes: no memory, barrier or TMEM effect.
+    // Warm-up while the predecessor finishes: no memory, barrier or TMEM effect
+    // (the top-k in the second epilogue group only).
     if (warp == 1 && lane == 0) {
         mma_kblock(0u, 0u, 0ull, 0ull, idesc_m128(kNTile), 1u);
-    } else if (warp >= 2 && warp < kBuildWarp) {
+    } else if (warp >= 2 + kGroupWarps && warp < kBuildWarp) {
         topk_item(zs, P, top_k, lane, 0, nullptr, nullptr);
     }
     // The work list is the predecessor's output (read with plain loads: a
