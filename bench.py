@@ -76,6 +76,9 @@ def parse():
     ap.add_argument("--level2-ctas", type=int, default=-1,
                     help="CTAs of level 2 in the replicated steps (-1: 56 with four or more streams, else one "
                          "per SM; 0: one per SM)")
+    ap.add_argument("--value-width", type=int, default=0,
+                    help="value row width d_v in place of the workload's (0: the workload's own); for ncu captures "
+                         "of level 2, which streams keys only, within a few GB of device memory")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle baseline")
     return ap.parse_args()
 
@@ -1069,6 +1072,8 @@ def main():
     from paper_2607_16305_gb300 import workloads as W
 
     w = W.WORKLOADS[args.workload]
+    if args.value_width > 0:
+        w = w.scaled(d_value=args.value_width)
     ws, rank, local = dist_env()
     if args.impl == "reference":
         if rank == 0:
