@@ -277,12 +277,15 @@ def test_lookup_inject_small_against_oracle(oracle, lookme_lib, name):
     run_case(oracle, lookme_lib, w, fused=True, n_layers=3 if name == "layers" else None)
 
 
-@pytest.mark.parametrize("P,dk,top_k", [(512, 256, 8), (384, 256, 8), (600, 128, 4), (1024, 64, 1), (264, 256, 8)])
+@pytest.mark.parametrize("P,dk,top_k", [(512, 256, 8), (384, 256, 8), (600, 128, 4), (1024, 64, 1), (264, 256, 8),
+                                          (1024, 512, 16)])
 def test_lookup_inject_ntile_topk(oracle, lookme_lib, P, dk, top_k):
     """Several N-tiles of primitives (MMAs of 256 keys each, a partial last one
     included: 600 = 2 x 256 + 88, 264 = 256 + 8) with small top-k, against the
-    oracle."""
-    w = W.small(f"ntile_{P}_{dk}_{top_k}", n_tokens=1500, n_scenes=60, n_prims=P, d_key=dk, d_value=128,
+    oracle; 1,024 x 512 with top-16 is the large-table shape, whose level-2
+    shared memory is the closest to the per-CTA limit."""
+    n_scenes = 20 if dk >= 512 else 60
+    w = W.small(f"ntile_{P}_{dk}_{top_k}", n_tokens=1500, n_scenes=n_scenes, n_prims=P, d_key=dk, d_value=128,
                 top_k=top_k, keep_ratio=0.25, n_segments=2, dtype="bf16")
     run_case(oracle, lookme_lib, w, fused=True)
 
